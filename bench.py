@@ -1,0 +1,362 @@
+#!/usr/bin/env python
+"""ES-iteration throughput of the CoPES core on GB300.
+
+Workload: 4B-parameter decoder-shaped set (36 layers, hidden 2560, MLP 9728, vocab 151936,
+tied embeddings; 4,022,468,096 parameters), bf16 working weights + fp32 master (24 GB
+resident), K = 8 layer-block subspaces, N = 32 antithetic members, sigma = 1e-3,
+alpha = 5e-4, z-score shaping, step coefficient alpha / (N sigma).
+
+One step = one cooperative-coevolution cycle: for each of the 8 subspaces, rebuild its
+tile table (the partition step), 32 perturbs (one per member; rewards are seeded
+synthetic scalars, no model is evaluated), restore, fitness shaping and the fused update
++ context commit.  Every parameter passes through 32 perturbs, one restore and one
+update per step, so value = parameters per step x steps / time.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl copes|reference]
+
+Prints one JSON line (rank 0).  Under torchrun each rank runs an independent replica on
+its own GPU (the path needs no exchange at this scope), timed with a barrier and the max
+over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "ES-iteration params/s and HBM GB/s at 4B bf16 (N=32), % of roofline on 1 GB300"
+FALLBACK_HBM_GBS = 6800.0
+
+# ncu DRAM bytes per element of the dominant kernel (perturb, bf16) from one capture; the
+# figure is dropped (traffic = null) when es_kernels.cu no longer matches the hash it
+# was taken on.
+NCU_TRAFFIC = {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": None, "bytes_per_elem": None}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="copes", choices=["copes", "reference"])
+    ap.add_argument("--tile", type=int, default=1 << 14)
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-sample", type=int, default=1 << 20,
+                    help="parameters of the oracle's timed CPU sample")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as fh:
+            return json.load(fh), "measured"
+    return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+def source_sha():
+    with open(os.path.join(ROOT, "paper_2608_02391_gb300", "csrc", "es_kernels.cu"), "rb") as fh:
+        a = fh.read()
+    with open(os.path.join(ROOT, "paper_2608_02391_gb300", "csrc", "copes_device.cuh"), "rb") as fh:
+        b = fh.read()
+    return hashlib.sha256(a + b).hexdigest()[:16]
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "lines", []):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ------------------------------------------------------------------------ CPU oracle leg
+def oracle_visit_sample(wl, n_sample: int, iteration: int = 0):
+    """The oracle as it stands on a bounded sample: one subspace visit (N perturbs,
+    restore, shaping, fused update + commit) restricted to the first n_sample parameters
+    of subspace 0.  Returns (seconds, parameters)."""
+    import oracle
+    from paper_2608_02391_gb300 import workloads
+    N = wl.n_members
+    rng = np.random.default_rng(0)
+    master = (rng.standard_normal(n_sample) * 0.02).astype(np.float32)
+    w = np.zeros(n_sample, np.uint16)
+    sub = oracle.make_subspace(ranges=[(0, n_sample)])
+    nid, sign, P = oracle.member_table(N, oracle.ANTITHETIC)
+    seeds = np.array([oracle.member_seed(wl.base_seed, iteration, 0, j) for j in range(P)], np.uint64)
+    rewards = workloads.reward_stream(wl, 1)[0]
+    t0 = time.perf_counter()
+    for i in range(N):
+        oracle.perturb(w, master, sub, int(seeds[nid[i]]), float(sign[i]) * wl.sigma)
+    oracle.restore(w, master, sub)
+    f = oracle.shape_fitness(rewards, oracle.SHAPE_ZSCORE)
+    coef = np.float32(oracle.step_coef(wl.alpha, N, wl.sigma, oracle.COEF_OPENAI))
+    oracle.update(master, sub, nid, sign, f, seeds, coef, w=w)
+    return time.perf_counter() - t0, n_sample
+
+
+def run_reference(args, wl):
+    rank, world, _ = dist_env()
+    if world > 1 and rank != 0:
+        return
+    import oracle
+    oracle.build()
+    n = max(1024, args.cpu_sample // 4)
+    for _ in range(max(args.warmup, 0)):
+        oracle_visit_sample(wl, 1024)
+    tot_t, tot_n = 0.0, 0
+    for s in range(args.steps):
+        t, m = oracle_visit_sample(wl, n, iteration=s)
+        tot_t += t
+        tot_n += m
+    value = tot_n / tot_t
+    sample = (f"each step: one subspace visit (N={wl.n_members} perturbs, restore, z-score shaping, "
+              f"fused update + commit) over {n} parameters, single thread")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / args.steps,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_config(wl, args),
+        "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "params/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def workload_config(wl, args):
+    return {"workload": "4B decoder-shaped bf16 set, fp32 master, K=8 layer blocks, N=32 antithetic",
+            "params": wl.d, "layers": 36, "hidden": 2560, "mlp": 9728, "vocab": 151936, "tied": True,
+            "K": wl.K, "N": wl.n_members, "sigma": wl.sigma, "alpha": wl.alpha, "shaping": wl.shaping,
+            "tile": args.tile, "l2": "inputs larger than L2 (24 GB resident per step), no flush"}
+
+
+# -------------------------------------------------------------------------- GPU leg
+def main():
+    args = parse()
+    from paper_2608_02391_gb300 import workloads
+    wl = workloads.workload("4b")
+    if args.impl == "reference":
+        return run_reference(args, wl)
+
+    import torch
+    from paper_2608_02391_gb300 import copes, es
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    copes.load()
+
+    layout = copes.Layout(wl.numel)
+    d = wl.d
+    master = torch.empty(layout.d_pad, dtype=torch.float32, device="cuda")
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(wl.init_seed)
+    master.normal_(0.0, wl.init_scale, generator=gen)  # seeded synthetic weights
+    offs = layout.offsets
+    for t, ten in enumerate(wl.tensors):
+        if ten.kind == "norm":
+            master[int(offs[t]):int(offs[t]) + ten.numel].fill_(1.0)
+    w = master.to(torch.bfloat16)
+    arena = copes.Arena(w, master)
+    cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping=wl.shaping)
+    total_steps = args.warmup + args.steps + args.e2e_steps
+    rewards_host = workloads.reward_stream(wl, total_steps * wl.K)  # [steps*K, N]
+    rewards_dev = torch.from_numpy(rewards_host).cuda()
+    fitness = torch.empty(wl.n_members, dtype=torch.float32, device="cuda")
+    spec_groups = np.ascontiguousarray(wl.group_of, np.int32)
+    subs = es.build_subspaces(layout, "groups", wl.K, group_of=wl.group_of, tile_size=args.tile)
+    tile_buf = [s.tensor for s in subs]
+
+    import ctypes
+    L = copes.load()
+
+    def rebuild(k):
+        """The partition step for subspace k: recompute its tile table into its buffer."""
+        spec = copes.PartitionSpec(copes.PART_TENSOR_GROUPS, wl.K, 0, 0,
+                                   spec_groups.ctypes.data_as(ctypes.c_void_p))
+        cnt = ctypes.c_uint64()
+        copes._check(L.copes_subspace_build(ctypes.byref(layout.desc), ctypes.byref(spec), k, args.tile, None,
+                                            ctypes.c_void_p(tile_buf[k].data_ptr()), tile_buf[k].shape[0],
+                                            ctypes.byref(cnt), copes._stream(None)))
+
+    def step(s, events=None):
+        for k in range(wl.K):
+            rebuild(k)
+            es.round_robin_visit(arena, subs[k], k, s, cfg, d, rewards_dev[s * wl.K + k],
+                                 fitness_out=fitness, events=events)
+
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    copes.check()
+    if world > 1:
+        dist.barrier()
+
+    events = {}
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        torch.cuda.synchronize()
+        start.record()
+        for s in range(args.warmup, args.warmup + args.steps):
+            step(s, events)
+        end.record()
+        torch.cuda.synchronize()
+    ms = start.elapsed_time(end)
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    copes.check()
+
+    # end to end through the public API: rewards from pinned host memory each visit,
+    # the shaped fitness read back each step, host wall clock
+    pinned = torch.from_numpy(rewards_host).pin_memory()
+    fit_host = torch.empty((wl.K, wl.n_members), dtype=torch.float32).pin_memory()
+    r_dev = torch.empty(wl.n_members, dtype=torch.float32, device="cuda")
+    f_all = torch.empty((wl.K, wl.n_members), dtype=torch.float32, device="cuda")
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    s0 = args.warmup + args.steps
+    for s in range(s0, s0 + args.e2e_steps):
+        for k in range(wl.K):
+            rebuild(k)
+            r_dev.copy_(pinned[s * wl.K + k], non_blocking=True)
+            es.round_robin_visit(arena, subs[k], k, s, cfg, d, r_dev, fitness_out=f_all[k])
+        fit_host.copy_(f_all, non_blocking=True)
+        torch.cuda.synchronize()
+    e2e_s = time.perf_counter() - t0
+    if world > 1:
+        t = torch.tensor([e2e_s], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_s = float(t.item())
+
+    if rank != 0:
+        dist.destroy_process_group() if world > 1 else None
+        return
+
+    # per-kernel average launch times (CUDA events on the launching stream)
+    per = {name: float(np.mean([a.elapsed_time(b) for a, b in lst])) for name, lst in events.items()}
+    counts = {name: len(lst) for name, lst in events.items()}
+    d_k = [s.numel for s in subs]
+    mean_dk = float(np.mean(d_k))
+    peaks, peak_src = measured_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    perturb_bytes = 6.0 * mean_dk
+    achieved = perturb_bytes / (per["perturb"] * 1e-3) / 1e9
+    traffic = None
+    if NCU_TRAFFIC["source_sha"] == source_sha() and NCU_TRAFFIC["bytes_per_elem"]:
+        traffic = NCU_TRAFFIC["bytes_per_elem"] * mean_dk
+    props = torch.cuda.get_device_properties(local)
+    clk = clocks.summary()
+    n_normals_update = wl.n_members // 2
+    alu_ops_per_normal = 28  # pinned algorithmic op count: 27 per normal + 1 fma
+    sm_mhz = clk["sm_mhz"] or float(peaks.get("sm_max_mhz", 2070.0))
+    alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12  # Tops/s at the sampled clock
+    upd_ops = mean_dk * n_normals_update * alu_ops_per_normal / (per["update"] * 1e-3) / 1e12
+    bytes_per_step = d * (wl.n_members * 6 + 6 + 10)
+    value = world * d * args.steps / (ms * 1e-3)
+    e2e = world * d * args.e2e_steps / e2e_s
+    launches = sum(counts.values())
+    out = {
+        "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": workload_config(wl, args),
+        "hbm_gbs": bytes_per_step * args.steps / (ms * 1e-3) / 1e9,
+        "roofline": {"bound": "hbm", "kernel": "perturb", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm, "traffic": traffic, "peak_source": peak_src,
+                     "algorithmic_bytes_per_launch": perturb_bytes},
+        "kernels": {
+            "perturb": {"ms": per["perturb"], "launches": counts["perturb"], "GB/s": achieved,
+                        "frac_hbm": achieved / hbm},
+            "restore": {"ms": per["restore"], "launches": counts["restore"],
+                        "GB/s": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9,
+                        "frac_hbm": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9 / hbm},
+            "update_fused_commit": {"ms": per["update"], "launches": counts["update"],
+                                    "GB/s": 10.0 * mean_dk / (per["update"] * 1e-3) / 1e9,
+                                    "bound": "alu", "achieved_Tops": upd_ops, "peak_Tops": alu_peak,
+                                    "frac_alu": upd_ops / alu_peak,
+                                    "ops_per_normal": alu_ops_per_normal, "normals_per_elem": n_normals_update},
+            "shape": {"ms": per["shape"], "launches": counts["shape"]},
+        },
+        "clocks": clk,
+        "e2e": {"value": e2e, "unit": "params/s", "h2d_bytes_per_step": wl.K * wl.n_members * 4,
+                "d2h_bytes_per_step": wl.K * wl.n_members * 4},
+        "gpu_launches": launches,
+    }
+    if not args.no_cpu_baseline and world == 1:
+        import oracle
+        oracle.build()
+        t, m = oracle_visit_sample(wl, args.cpu_sample)
+        out["cpu_baseline"] = {
+            "value": m / t, "unit": "params/s", "cores": 1, "kind": "oracle",
+            "sample": f"one subspace visit (N={wl.n_members} perturbs, restore, shaping, fused update + "
+                      f"commit) over {m} parameters of subspace 0, single thread, {t:.1f} s"}
+    print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,340 @@
+"""Thin ctypes binding of libcopes.so (the C ABI in include/copes.h).
+
+Argument marshalling only: torch supplies device memory and streams, every step runs in
+the library's CUDA kernels.  The names follow the C ABI.  Loading fails loudly when the
+library has not been built; there is no fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import List, Optional, Sequence
+
+import numpy as np
+import torch
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libcopes.so")
+
+OK = 0
+ERR_INVALID_ARG, ERR_ALIGNMENT, ERR_SIZE, ERR_WORKSPACE, ERR_CUDA, ERR_DEVICE_CHECK, ERR_UNSUPPORTED = \
+    -1, -2, -3, -4, -5, -6, -7
+BF16, FP32 = 0, 1
+TAG_NOISE, TAG_INIT, TAG_PARTITION, TAG_SEED, TAG_CHUNK = 0, 1, 2, 3, 4
+MAX_MEMBERS, MAX_NOISE, MAX_K, TILE_MAX = 256, 256, 64, 1 << 20
+SUBSPACE_TILES, SUBSPACE_INDICES = 0, 1
+PART_CONTIGUOUS, PART_TENSOR_GROUPS, PART_HASH, PART_RANDOM_CHUNKS = 0, 1, 2, 3
+SHAPE_NONE, SHAPE_ZSCORE, SHAPE_ZSCORE_GROUPED, SHAPE_CENTERED_RANK = 0, 1, 2, 3
+ONE_SIDED, ANTITHETIC = 0, 1
+COEF_PAPER, COEF_OPENAI = 0, 1
+DEFAULT_TILE = 1 << 14
+
+SHAPE_MODES = {"none": SHAPE_NONE, "zscore": SHAPE_ZSCORE, "zscore_grouped": SHAPE_ZSCORE_GROUPED,
+               "centered_rank": SHAPE_CENTERED_RANK}
+
+
+class CopesError(RuntimeError):
+    def __init__(self, code: int, message: str):
+        super().__init__(f"[{code}] {message}")
+        self.code = code
+
+
+class Params(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("master", ctypes.c_void_p), ("n_alloc", ctypes.c_uint64),
+                ("dtype", ctypes.c_int)]
+
+
+class Subspace(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int), ("tiles", ctypes.c_void_p), ("n_tiles", ctypes.c_uint64),
+                ("index", ctypes.c_void_p), ("n_index", ctypes.c_uint64)]
+
+
+class LayoutDesc(ctypes.Structure):
+    _fields_ = [("n_tensors", ctypes.c_int), ("numel", ctypes.c_void_p), ("tensor_id", ctypes.c_void_p)]
+
+
+class PartitionSpec(ctypes.Structure):
+    _fields_ = [("mode", ctypes.c_int), ("K", ctypes.c_int), ("seed", ctypes.c_uint64),
+                ("chunk", ctypes.c_uint64), ("group_of", ctypes.c_void_p)]
+
+
+_lib = None
+
+# name -> (restype, argtypes); every function declared in include/copes.h.
+_VP, _U64, _U32, _I32, _F32, _F64, _SZ = (ctypes.c_void_p, ctypes.c_uint64, ctypes.c_uint32,
+                                          ctypes.c_int, ctypes.c_float, ctypes.c_double,
+                                          ctypes.c_size_t)
+SIGNATURES = {
+    "copes_version": (ctypes.c_char_p, []),
+    "copes_last_error": (_I32, [_VP, _SZ]),
+    "copes_check": (_I32, [_VP]),
+    "copes_layout": (_I32, [_VP, _VP]),
+    "copes_sigma_eff": (_F64, [_F64, _F64, _F64, _I32]),
+    "copes_step_coef": (_F64, [_F64, _I32, _F64, _I32]),
+    "copes_member_table": (_I32, [_I32, _I32, _VP, _VP]),
+    "copes_member_seed": (_U64, [_U64, _U32, _U32, _U32]),
+    "copes_subspace_build": (_I32, [_VP, _VP, _I32, _U64, _VP, _VP, _U64, _VP, _VP]),
+    "copes_tiles_from_ranges": (_I32, [_VP, _VP, _I32, _U64, _VP, _U64, _VP, _VP]),
+    "copes_random_chunk_map": (_I32, [_U64, _I32, _U64, _VP, _VP]),
+    "copes_hash_workspace_bytes": (_SZ, [_VP, _I32]),
+    "copes_hash_count": (_I32, [_VP, _I32, _U64, _VP, _SZ, _VP, _VP]),
+    "copes_hash_fill": (_I32, [_VP, _I32, _U64, _VP, _SZ, _VP, _VP]),
+    "copes_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
+    "copes_restore": (_I32, [_VP, _VP, _VP]),
+    "copes_context_commit": (_I32, [_VP, _VP, _VP]),
+    "copes_shape_fitness": (_I32, [_VP, _I32, _VP, _I32, _VP, _VP]),
+    "copes_update": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _F32, _I32, _VP]),
+    "copes_init_normal": (_I32, [_VP, _VP, _U64, _F32, _F32, _VP]),
+    "copes_debug_philox": (_I32, [_U64, _U64, _U64, _U32, _U32, _VP, _VP]),
+    "copes_debug_normals": (_I32, [_U64, _U32, _U64, _U64, _VP, _VP]),
+    "copes_debug_transform": (_I32, [_VP, _U64, _VP, _VP]),
+}
+
+
+def load():
+    """Load libcopes.so (raises if it is missing: build it with __graft_entry__.build())."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is missing: build the CUDA library first "
+                               "(python -c 'import __graft_entry__ as g; g.build()')")
+        lib = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+    return _lib
+
+
+def last_error() -> str:
+    buf = ctypes.create_string_buffer(1024)
+    load().copes_last_error(buf, len(buf))
+    return buf.value.decode()
+
+
+def _check(rc: int) -> int:
+    if rc < 0:
+        raise CopesError(rc, last_error())
+    return rc
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _np_ptr(a: Optional[np.ndarray]):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+# ------------------------------------------------------------------------ host helpers
+def version() -> str:
+    return load().copes_version().decode()
+
+
+def check(stream=None) -> None:
+    """Synchronise the stream and raise if a kernel's range check fired."""
+    _check(load().copes_check(_stream(stream)))
+
+
+def sigma_eff(sigma: float, d: float, d_k: float, dimension_aware: bool = True) -> float:
+    return load().copes_sigma_eff(sigma, float(d), float(d_k), int(dimension_aware))
+
+
+def step_coef(alpha: float, n_members: int, sigma_eff_: float, convention: int) -> float:
+    return load().copes_step_coef(alpha, n_members, sigma_eff_, convention)
+
+
+def member_table(n_members: int, pairing: int):
+    nid = np.zeros(n_members, np.int32)
+    sign = np.zeros(n_members, np.int8)
+    P = _check(load().copes_member_table(n_members, pairing, _np_ptr(nid), _np_ptr(sign)))
+    return nid, sign, P
+
+
+def member_seed(base_seed: int, iteration: int, k: int, j: int) -> int:
+    return int(load().copes_member_seed(base_seed, iteration, k, j))
+
+
+def member_seeds(base_seed: int, iteration: int, k: int, n_noise: int) -> np.ndarray:
+    return np.array([member_seed(base_seed, iteration, k, j) for j in range(n_noise)], np.uint64)
+
+
+class Layout:
+    """Host view of a tensor table (copes_layout_desc); keeps its arrays alive."""
+
+    def __init__(self, numel: Sequence[int], tensor_id: Optional[Sequence[int]] = None):
+        self.numel = np.ascontiguousarray(numel, dtype=np.uint64)
+        self.tensor_id = None if tensor_id is None else np.ascontiguousarray(tensor_id, np.uint32)
+        self.desc = LayoutDesc(self.numel.size, _np_ptr(self.numel), _np_ptr(self.tensor_id))
+        self.offsets = np.zeros(self.numel.size + 1, np.uint64)
+        _check(load().copes_layout(ctypes.byref(self.desc), _np_ptr(self.offsets)))
+
+    @property
+    def d_pad(self) -> int:
+        return int(self.offsets[-1])
+
+
+# ----------------------------------------------------------------------------- arena
+class Arena:
+    """The flat parameter arena: working weights w (bf16 or fp32) and the fp32 master."""
+
+    def __init__(self, w: torch.Tensor, master: torch.Tensor):
+        assert w.is_cuda and master.is_cuda and w.is_contiguous() and master.is_contiguous()
+        assert master.dtype == torch.float32 and w.numel() == master.numel()
+        self.w, self.master = w, master
+        dt = {torch.bfloat16: BF16, torch.float32: FP32}[w.dtype]
+        self.params = Params(w.data_ptr(), master.data_ptr(), w.numel(), dt)
+
+    @classmethod
+    def empty(cls, n: int, dtype=torch.bfloat16, device="cuda"):
+        return cls(torch.empty(n, dtype=dtype, device=device), torch.empty(n, dtype=torch.float32, device=device))
+
+    @property
+    def n_alloc(self) -> int:
+        return self.w.numel()
+
+
+@dataclass
+class SubspaceHandle:
+    """A subspace: device tiles ([n, 2] int64 holding uint64 bounds) or a device index list."""
+    kind: int
+    tensor: torch.Tensor
+    numel: int
+
+    def struct(self) -> Subspace:
+        if self.kind == SUBSPACE_TILES:
+            return Subspace(SUBSPACE_TILES, self.tensor.data_ptr() if self.tensor.numel() else None,
+                            self.tensor.shape[0], None, 0)
+        return Subspace(SUBSPACE_INDICES, None, 0,
+                        self.tensor.data_ptr() if self.tensor.numel() else None, self.tensor.numel())
+
+
+def _tiles_result(count_fn, fill_fn, device, stream) -> SubspaceHandle:
+    count = ctypes.c_uint64(0)
+    _check(count_fn(ctypes.byref(count)))
+    n = int(count.value)
+    tiles = torch.empty((max(n, 1), 2), dtype=torch.int64, device=device)
+    _check(fill_fn(tiles, n, ctypes.byref(count)))
+    t = tiles[:n]
+    numel = int((t[:, 1] - t[:, 0]).sum().item()) if n else 0
+    return SubspaceHandle(SUBSPACE_TILES, t, numel)
+
+
+def tiles_from_ranges(ranges, tile_size: int = DEFAULT_TILE, device="cuda", stream=None) -> SubspaceHandle:
+    b = np.ascontiguousarray([r[0] for r in ranges], np.uint64)
+    e = np.ascontiguousarray([r[1] for r in ranges], np.uint64)
+    L, s = load(), _stream(stream)
+    return _tiles_result(
+        lambda cnt: L.copes_tiles_from_ranges(_np_ptr(b), _np_ptr(e), len(ranges), tile_size, None, 0, cnt, s),
+        lambda t, n, cnt: L.copes_tiles_from_ranges(_np_ptr(b), _np_ptr(e), len(ranges), tile_size,
+                                                    _ptr(t), n, cnt, s), device, stream)
+
+
+def subspace_build(layout: Layout, mode: int, K: int, k: int, seed: int = 0, chunk: int = 65536,
+                   group_of: Optional[Sequence[int]] = None, chunk_map: Optional[torch.Tensor] = None,
+                   tile_size: int = DEFAULT_TILE, device="cuda", stream=None) -> SubspaceHandle:
+    """copes_subspace_build for the range modes (CONTIGUOUS, TENSOR_GROUPS, RANDOM_CHUNKS)."""
+    g = None if group_of is None else np.ascontiguousarray(group_of, np.int32)
+    spec = PartitionSpec(mode, K, seed, chunk, _np_ptr(g))
+    L, s = load(), _stream(stream)
+    cm = _ptr(chunk_map)
+    return _tiles_result(
+        lambda cnt: L.copes_subspace_build(ctypes.byref(layout.desc), ctypes.byref(spec), k, tile_size,
+                                           cm, None, 0, cnt, s),
+        lambda t, n, cnt: L.copes_subspace_build(ctypes.byref(layout.desc), ctypes.byref(spec), k,
+                                                 tile_size, cm, _ptr(t), n, cnt, s), device, stream)
+
+
+def random_chunk_map(n_chunks: int, K: int, seed: int, device="cuda", stream=None) -> torch.Tensor:
+    out = torch.empty(n_chunks, dtype=torch.int32, device=device)
+    _check(load().copes_random_chunk_map(n_chunks, K, seed, _ptr(out), _stream(stream)))
+    return out
+
+
+def hash_partition(layout: Layout, K: int, seed: int, device="cuda", stream=None) -> List[SubspaceHandle]:
+    """copes_hash_count + copes_hash_fill: K sorted int64 index lists (torch-allocated)."""
+    L, s = load(), _stream(stream)
+    nbytes = L.copes_hash_workspace_bytes(ctypes.byref(layout.desc), K)
+    if nbytes == 0:
+        raise CopesError(ERR_INVALID_ARG, "copes_hash_workspace_bytes rejected the layout / K")
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=device)
+    counts = np.zeros(K, np.uint64)
+    _check(L.copes_hash_count(ctypes.byref(layout.desc), K, seed, _ptr(ws), nbytes, _np_ptr(counts), s))
+    lists = [torch.empty(max(int(c), 2), dtype=torch.int64, device=device) for c in counts]
+    ptrs = (ctypes.c_void_p * K)(*[t.data_ptr() for t in lists])
+    _check(L.copes_hash_fill(ctypes.byref(layout.desc), K, seed, _ptr(ws), nbytes, ptrs, s))
+    if stream is not None:
+        ws.record_stream(stream)  # freed in stream order with the fill's kernels
+    return [SubspaceHandle(SUBSPACE_INDICES, t[:int(c)], int(c)) for t, c in zip(lists, counts)]
+
+
+# -------------------------------------------------------------------------- ES steps
+def perturb(arena: Arena, sub: SubspaceHandle, seed: int, signed_sigma: float, stream=None) -> None:
+    S = sub.struct()
+    _check(load().copes_perturb(ctypes.byref(arena.params), ctypes.byref(S), seed, signed_sigma, _stream(stream)))
+
+
+def restore(arena: Arena, sub: SubspaceHandle, stream=None) -> None:
+    S = sub.struct()
+    _check(load().copes_restore(ctypes.byref(arena.params), ctypes.byref(S), _stream(stream)))
+
+
+def context_commit(arena: Arena, sub: SubspaceHandle, stream=None) -> None:
+    S = sub.struct()
+    _check(load().copes_context_commit(ctypes.byref(arena.params), ctypes.byref(S), _stream(stream)))
+
+
+def init_normal(arena: Arena, sub: SubspaceHandle, seed: int, mean: float, scale: float, stream=None) -> None:
+    S = sub.struct()
+    _check(load().copes_init_normal(ctypes.byref(arena.params), ctypes.byref(S), seed, mean, scale,
+                                    _stream(stream)))
+
+
+def shape_fitness(rewards: torch.Tensor, mode, group: Optional[torch.Tensor] = None,
+                  out: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    mode = SHAPE_MODES[mode] if isinstance(mode, str) else mode
+    assert rewards.dtype == torch.float32 and rewards.is_cuda and rewards.is_contiguous()
+    if out is None:
+        out = torch.empty_like(rewards)
+    _check(load().copes_shape_fitness(_ptr(rewards), rewards.numel(), _ptr(group), mode, _ptr(out),
+                                      _stream(stream)))
+    return out
+
+
+def update(arena: Arena, sub: SubspaceHandle, noise_id: np.ndarray, sign: np.ndarray,
+           fitness: torch.Tensor, seeds: np.ndarray, coef: float, fuse_commit: bool = True,
+           stream=None) -> None:
+    nid = np.ascontiguousarray(noise_id, np.int32)
+    sg = np.ascontiguousarray(sign, np.int8)
+    sd = np.ascontiguousarray(seeds, np.uint64)
+    S = sub.struct()
+    _check(load().copes_update(ctypes.byref(arena.params), ctypes.byref(S), nid.size, _np_ptr(nid),
+                               _np_ptr(sg), _ptr(fitness), sd.size, _np_ptr(sd), coef,
+                               int(fuse_commit), _stream(stream)))
+
+
+# ----------------------------------------------------------------------------- debug
+def debug_philox(seed: int, q0: int, n: int, aux: int = 0, tag: int = TAG_NOISE, stream=None) -> torch.Tensor:
+    out = torch.empty(4 * n, dtype=torch.int32, device="cuda")
+    _check(load().copes_debug_philox(seed, q0, n, aux, tag, _ptr(out), _stream(stream)))
+    return out
+
+
+def debug_normals(seed: int, g0: int, n: int, tag: int = TAG_NOISE, stream=None) -> torch.Tensor:
+    out = torch.empty(n, dtype=torch.float32, device="cuda")
+    _check(load().copes_debug_normals(seed, tag, g0, n, _ptr(out), _stream(stream)))
+    return out
+
+
+def debug_transform(words: torch.Tensor, stream=None) -> torch.Tensor:
+    out = torch.empty(words.numel(), dtype=torch.float32, device=words.device)
+    _check(load().copes_debug_transform(_ptr(words), words.numel(), _ptr(out), _stream(stream)))
+    return out

@@ -1,0 +1,128 @@
+// Internal declarations shared by the host API and the kernel translation units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/copes.h"
+
+namespace copes {
+
+constexpr int kThreads = 256;       // threads per block of the elementwise kernels
+constexpr int kIndexSegment = 8192; // indices per block in the gather kernels
+
+// Philox4x32-10 constants (SC'11, Sec. 3): round multipliers and key (Weyl) increments.
+constexpr uint32_t kPhiloxM0 = 0xD2511F53u;
+constexpr uint32_t kPhiloxM1 = 0xCD9E8D57u;
+constexpr uint32_t kPhiloxW0 = 0x9E3779B9u;
+constexpr uint32_t kPhiloxW1 = 0xBB67AE85u;
+
+// Philox4x32-10 on one counter: 10 rounds of (two 32x32->64 multiplies, XOR of the high
+// halves with the other counter words and the round key, key bump).  Host and device.
+__host__ __device__ __forceinline__ void philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2,
+                                                       uint32_t c3, uint32_t k0, uint32_t k1,
+                                                       uint32_t out[4]) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint64_t p0 = (uint64_t)kPhiloxM0 * c0;
+    const uint64_t p1 = (uint64_t)kPhiloxM1 * c2;
+    const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ k0;
+    const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ k1;
+    c1 = (uint32_t)p1;
+    c3 = (uint32_t)p0;
+    c0 = n0;
+    c2 = n2;
+    k0 += kPhiloxW0;
+    k1 += kPhiloxW1;
+  }
+  out[0] = c0;
+  out[1] = c1;
+  out[2] = c2;
+  out[3] = c3;
+}
+
+// Device error bits (set with atomicOr by a kernel that skipped an access).
+enum : unsigned {
+  kErrTileRange = 1u,   // a tile outside [0, n_alloc) or longer than COPES_TILE_MAX
+  kErrIndexRange = 2u,  // a gather index outside [0, n_alloc)
+  kErrPartition = 4u    // a partition kernel met an inconsistent workspace
+};
+
+// ---------------------------------------------------------------- launch arguments
+struct ElemArgs {
+  void *w;
+  float *master;
+  uint64_t n_alloc;
+  const uint64_t *tiles;
+  uint64_t n_tiles;
+  const int64_t *index;
+  uint64_t n_index;
+  uint32_t seed_lo, seed_hi;
+  uint32_t tag;
+  float a;  // perturb: signed sigma; init: scale
+  float b;  // init: mean
+};
+
+enum ElemOp { kOpPerturb = 0, kOpRestore = 1, kOpInit = 2 };
+
+struct UpdateArgs {
+  void *w;
+  float *master;
+  uint64_t n_alloc;
+  const uint64_t *tiles;
+  uint64_t n_tiles;
+  const int64_t *index;
+  uint64_t n_index;
+  const float *fitness;
+  float coef;
+  int n_members;
+  int n_noise;
+  int fuse_commit;
+  uint32_t seed_lo[COPES_MAX_NOISE];
+  uint32_t seed_hi[COPES_MAX_NOISE];
+  uint16_t noise_ptr[COPES_MAX_NOISE + 1];  // members of noise j: noise_member[ptr[j] .. ptr[j+1])
+  uint16_t noise_member[COPES_MAX_MEMBERS];
+  int8_t sign[COPES_MAX_MEMBERS];
+};
+
+// ------------------------------------------------------------------------ launchers
+// Each returns the launch's cudaError_t (cudaSuccess when nothing was launched).
+cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, cudaStream_t s);
+cudaError_t launch_update(int kind, int dtype, const UpdateArgs &a, cudaStream_t s,
+                          int num_sms);
+cudaError_t launch_shape(const float *r, int n, const int32_t *group, int mode, float *f,
+                         cudaStream_t s);
+cudaError_t launch_debug_philox(uint64_t seed, uint64_t q0, uint64_t n, uint32_t aux,
+                                uint32_t tag, uint32_t *out, cudaStream_t s);
+cudaError_t launch_debug_normals(uint64_t seed, uint32_t tag, uint64_t g0, uint64_t n,
+                                 float *out, cudaStream_t s);
+cudaError_t launch_debug_transform(const uint32_t *words, uint64_t n, float *out,
+                                   cudaStream_t s);
+
+// Hash partition.  The workspace begins with a table of HashTensor entries, then per
+// hash tile a K-bucket histogram (uint32), then per hash tile K exclusive offsets
+// (uint64), then K totals (unsigned long long).
+constexpr uint64_t kHashTile = 16384;
+struct HashTensor {
+  uint64_t offset;      // global offset of the tensor
+  uint64_t numel;
+  uint64_t tile_begin;  // first hash tile of the tensor
+  uint32_t tensor_id;
+  uint32_t pad;
+};
+cudaError_t launch_hash_hist(const HashTensor *tensors, int n_tensors, uint64_t n_htiles, int K,
+                             uint64_t seed, uint32_t *hist, unsigned long long *totals,
+                             cudaStream_t s);
+cudaError_t launch_hash_scan(const uint32_t *hist, uint64_t n_htiles, int K, uint64_t *offsets,
+                             cudaStream_t s);
+cudaError_t launch_hash_scatter(const HashTensor *tensors, int n_tensors, uint64_t n_htiles,
+                                int K, uint64_t seed, const uint64_t *offsets,
+                                int64_t *const *lists, cudaStream_t s);
+cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,
+                                    cudaStream_t s);
+
+// Device error words of each translation unit: read and clear (synchronous).
+unsigned read_and_clear_es_errors();
+unsigned read_and_clear_partition_errors();
+
+}  // namespace copes

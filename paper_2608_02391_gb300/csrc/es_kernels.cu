@@ -1,0 +1,400 @@
+// Elementwise ES kernels: perturb (Eq. 8), restore / context commit (Supp. A.8), the
+// fused reward-weighted update (Eq. 6 / Eq. 13) and the synthetic initialiser, over
+// TILES subspaces (vectorised, 4-element groups = one Philox counter) and INDICES
+// subspaces (gather / scatter through a sorted int64 list).
+#include <cuda_bf16.h>
+
+#include "copes_device.cuh"
+#include "copes_internal.h"
+
+namespace copes {
+
+__device__ unsigned int g_es_error = 0;
+
+__device__ __forceinline__ void flag_error(unsigned bit) { atomicOr(&g_es_error, bit); }
+
+// ----------------------------------------------------------------- group primitives
+// A "group" is the 4 consecutive global indices 4q .. 4q+3, which share Philox counter q.
+
+template <typename WT>
+struct WStore;
+
+template <>
+struct WStore<__nv_bfloat16> {
+  static __device__ __forceinline__ void full(void *w, uint64_t g, const float v[4]) {
+    uint2 p;
+    p.x = pack_bf16x2(v[0], v[1]);
+    p.y = pack_bf16x2(v[2], v[3]);
+    st_stream_u2(reinterpret_cast<uint16_t *>(w) + g, p);
+  }
+  static __device__ __forceinline__ void one(void *w, uint64_t g, float v) {
+    reinterpret_cast<uint16_t *>(w)[g] = to_bf16_bits(v);
+  }
+};
+
+template <>
+struct WStore<float> {
+  static __device__ __forceinline__ void full(void *w, uint64_t g, const float v[4]) {
+    st_stream_f4(reinterpret_cast<float *>(w) + g, make_float4(v[0], v[1], v[2], v[3]));
+  }
+  static __device__ __forceinline__ void one(void *w, uint64_t g, float v) {
+    reinterpret_cast<float *>(w)[g] = v;
+  }
+};
+
+// Noise for the group at 4q under (k0, k1, tag): four normals.
+__device__ __forceinline__ void group_noise(uint64_t q, uint32_t tag, uint32_t k0, uint32_t k1,
+                                            float eps[4]) {
+  uint32_t x[4];
+  philox4x32_10((uint32_t)q, (uint32_t)(q >> 32), 0u, tag, k0, k1, x);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) eps[e] = normal_from_word(x[e]);
+}
+
+// Noise for a single index g: the one word of its counter that g uses.
+__device__ __forceinline__ float index_noise(uint64_t g, uint32_t tag, uint32_t k0, uint32_t k1) {
+  uint32_t x[4];
+  const uint64_t q = g >> 2;
+  philox4x32_10((uint32_t)q, (uint32_t)(q >> 32), 0u, tag, k0, k1, x);
+  const uint32_t s = (uint32_t)g & 3u;
+  const uint32_t w = s == 0 ? x[0] : (s == 1 ? x[1] : (s == 2 ? x[2] : x[3]));
+  return normal_from_word(w);
+}
+
+// ------------------------------------------------------------ perturb / restore / init
+template <int OP>
+__device__ __forceinline__ void elem_values(const ElemArgs &a, uint64_t g4, const float th[4],
+                                            float v[4]) {
+  if (OP == kOpRestore) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) v[e] = th[e];
+  } else {
+    float eps[4];
+    group_noise(g4 >> 2, a.tag, a.seed_lo, a.seed_hi, eps);
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      v[e] = (OP == kOpPerturb) ? __fmaf_rn(a.a, eps[e], th[e]) : __fmaf_rn(a.a, eps[e], a.b);
+  }
+}
+
+template <int OP, typename WT, int G>
+__global__ void __launch_bounds__(kThreads) elem_tiles_kernel(const ElemArgs a) {
+  const uint64_t t = blockIdx.x;
+  const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
+  if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
+    if (threadIdx.x == 0) flag_error(kErrTileRange);
+    return;
+  }
+  float *__restrict__ master = a.master;
+  const uint64_t lo = b & ~3ull;
+  for (uint64_t base = lo + 4ull * threadIdx.x; base < e; base += 4ull * kThreads * G) {
+    float th[G][4];
+    bool full[G];
+#pragma unroll
+    for (int i = 0; i < G; ++i) {
+      const uint64_t g4 = base + 4ull * kThreads * i;
+      full[i] = g4 >= b && g4 + 4 <= e;
+      if (OP != kOpInit) {
+        if (full[i]) {
+          const float4 v = ld_stream_f4(master + g4);
+          th[i][0] = v.x, th[i][1] = v.y, th[i][2] = v.z, th[i][3] = v.w;
+        } else {
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            th[i][k] = (g4 + k >= b && g4 + k < e) ? master[g4 + k] : 0.0f;
+        }
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) th[i][k] = 0.0f;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < G; ++i) {
+      const uint64_t g4 = base + 4ull * kThreads * i;
+      if (g4 >= e) continue;
+      float v[4];
+      elem_values<OP>(a, g4, th[i], v);
+      if (full[i]) {
+        if (OP == kOpInit) st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
+        WStore<WT>::full(a.w, g4, v);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const uint64_t g = g4 + k;
+          if (g >= b && g < e) {
+            if (OP == kOpInit) master[g] = v[k];
+            WStore<WT>::one(a.w, g, v[k]);
+          }
+        }
+      }
+    }
+  }
+}
+
+template <int OP, typename WT>
+__global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) {
+  constexpr int U = 4;
+  const uint64_t s0 = (uint64_t)blockIdx.x * kIndexSegment;
+  const uint64_t s1 = min(s0 + (uint64_t)kIndexSegment, a.n_index);
+  float *__restrict__ master = a.master;
+  for (uint64_t i0 = s0 + threadIdx.x; i0 < s1; i0 += (uint64_t)kThreads * U) {
+    int64_t g[U];
+    float th[U];
+    bool ok[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint64_t i = i0 + (uint64_t)kThreads * u;
+      ok[u] = i < s1;
+      g[u] = ok[u] ? a.index[i] : 0;
+      if (ok[u] && (g[u] < 0 || (uint64_t)g[u] >= a.n_alloc)) {
+        flag_error(kErrIndexRange);
+        ok[u] = false;
+      }
+      th[u] = (OP != kOpInit && ok[u]) ? master[g[u]] : 0.0f;
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (!ok[u]) continue;
+      float v;
+      if (OP == kOpRestore) {
+        v = th[u];
+      } else {
+        const float eps = index_noise((uint64_t)g[u], a.tag, a.seed_lo, a.seed_hi);
+        v = (OP == kOpPerturb) ? __fmaf_rn(a.a, eps, th[u]) : __fmaf_rn(a.a, eps, a.b);
+      }
+      if (OP == kOpInit) master[g[u]] = v;
+      WStore<WT>::one(a.w, (uint64_t)g[u], v);
+    }
+  }
+}
+
+template <int OP, typename WT>
+static cudaError_t launch_elem_typed(int kind, const ElemArgs &a, cudaStream_t s) {
+  if (kind == COPES_SUBSPACE_TILES) {
+    if (a.n_tiles == 0) return cudaSuccess;
+    constexpr int G = (OP == kOpRestore) ? 4 : 2;
+    elem_tiles_kernel<OP, WT, G><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+  } else {
+    if (a.n_index == 0) return cudaSuccess;
+    const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
+    elem_index_kernel<OP, WT><<<(unsigned)blocks, kThreads, 0, s>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+template <int OP>
+static cudaError_t launch_elem_op(int kind, int dtype, const ElemArgs &a, cudaStream_t s) {
+  return dtype == COPES_BF16 ? launch_elem_typed<OP, __nv_bfloat16>(kind, a, s)
+                             : launch_elem_typed<OP, float>(kind, a, s);
+}
+
+cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, cudaStream_t s) {
+  switch (op) {
+    case kOpPerturb: return launch_elem_op<kOpPerturb>(kind, dtype, a, s);
+    case kOpRestore: return launch_elem_op<kOpRestore>(kind, dtype, a, s);
+    default: return launch_elem_op<kOpInit>(kind, dtype, a, s);
+  }
+}
+
+// ------------------------------------------------------------------------- update
+// One block per tile.  The prologue folds the members into one weight per noise vector,
+//   w_j = sum_{i : noise(i) = j} sign_i f_i  (member order, fp32),
+// then every thread regenerates all P noise vectors for its groups in registers and
+// accumulates acc = sum_j w_j eps_j (j ascending), theta = fma(coef, acc, theta).
+__device__ __forceinline__ void noise_weights_to_smem(const UpdateArgs &a, float *s_w) {
+  for (int j = threadIdx.x; j < a.n_noise; j += blockDim.x) {
+    float acc = 0.0f;
+    for (int m = a.noise_ptr[j]; m < a.noise_ptr[j + 1]; ++m) {
+      const int i = a.noise_member[m];
+      const float f = a.fitness[i];
+      acc = __fadd_rn(acc, a.sign[i] > 0 ? f : -f);
+    }
+    s_w[j] = acc;
+  }
+  __syncthreads();
+}
+
+template <typename WT, int G, bool COMMIT>
+__global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
+  __shared__ float s_w[COPES_MAX_NOISE];
+  noise_weights_to_smem(a, s_w);
+  const uint64_t t = blockIdx.x;
+  const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
+  if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
+    if (threadIdx.x == 0) flag_error(kErrTileRange);
+    return;
+  }
+  float *__restrict__ master = a.master;
+  const uint64_t lo = b & ~3ull;
+  const int P = a.n_noise;
+  for (uint64_t base = lo + 4ull * threadIdx.x; base < e; base += 4ull * kThreads * G) {
+    float th[G][4], acc[G][4];
+    bool full[G];
+#pragma unroll
+    for (int i = 0; i < G; ++i) {
+      const uint64_t g4 = base + 4ull * kThreads * i;
+      full[i] = g4 >= b && g4 + 4 <= e;
+      if (full[i]) {
+        const float4 v = ld_stream_f4(master + g4);
+        th[i][0] = v.x, th[i][1] = v.y, th[i][2] = v.z, th[i][3] = v.w;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          th[i][k] = (g4 + k >= b && g4 + k < e) ? master[g4 + k] : 0.0f;
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) acc[i][k] = 0.0f;
+    }
+    for (int j = 0; j < P; ++j) {
+      const uint32_t k0 = a.seed_lo[j], k1 = a.seed_hi[j];
+      const float wj = s_w[j];
+#pragma unroll
+      for (int i = 0; i < G; ++i) {
+        float eps[4];
+        group_noise((base + 4ull * kThreads * i) >> 2, COPES_TAG_NOISE, k0, k1, eps);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < G; ++i) {
+      const uint64_t g4 = base + 4ull * kThreads * i;
+      if (g4 >= e) continue;
+      float v[4];
+#pragma unroll
+      for (int k = 0; k < 4; ++k) v[k] = __fmaf_rn(a.coef, acc[i][k], th[i][k]);
+      if (full[i]) {
+        st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
+        if (COMMIT) WStore<WT>::full(a.w, g4, v);
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const uint64_t g = g4 + k;
+          if (g >= b && g < e) {
+            master[g] = v[k];
+            if (COMMIT) WStore<WT>::one(a.w, g, v[k]);
+          }
+        }
+      }
+    }
+  }
+}
+
+template <typename WT, bool COMMIT>
+__global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_constant__ UpdateArgs a) {
+  __shared__ float s_w[COPES_MAX_NOISE];
+  noise_weights_to_smem(a, s_w);
+  constexpr int U = 2;
+  const uint64_t s0 = (uint64_t)blockIdx.x * kIndexSegment;
+  const uint64_t s1 = min(s0 + (uint64_t)kIndexSegment, a.n_index);
+  float *__restrict__ master = a.master;
+  const int P = a.n_noise;
+  for (uint64_t i0 = s0 + threadIdx.x; i0 < s1; i0 += (uint64_t)kThreads * U) {
+    int64_t g[U];
+    float th[U], acc[U];
+    bool ok[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      const uint64_t i = i0 + (uint64_t)kThreads * u;
+      ok[u] = i < s1;
+      g[u] = ok[u] ? a.index[i] : 0;
+      if (ok[u] && (g[u] < 0 || (uint64_t)g[u] >= a.n_alloc)) {
+        flag_error(kErrIndexRange);
+        ok[u] = false;
+      }
+      th[u] = ok[u] ? master[g[u]] : 0.0f;
+      acc[u] = 0.0f;
+    }
+    for (int j = 0; j < P; ++j) {
+      const uint32_t k0 = a.seed_lo[j], k1 = a.seed_hi[j];
+      const float wj = s_w[j];
+#pragma unroll
+      for (int u = 0; u < U; ++u)
+        acc[u] = __fmaf_rn(wj, index_noise((uint64_t)g[u], COPES_TAG_NOISE, k0, k1), acc[u]);
+    }
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (!ok[u]) continue;
+      const float v = __fmaf_rn(a.coef, acc[u], th[u]);
+      master[g[u]] = v;
+      if (COMMIT) WStore<WT>::one(a.w, (uint64_t)g[u], v);
+    }
+  }
+}
+
+template <typename WT, bool COMMIT>
+static cudaError_t launch_update_typed(int kind, const UpdateArgs &a, cudaStream_t s) {
+  if (kind == COPES_SUBSPACE_TILES) {
+    if (a.n_tiles == 0) return cudaSuccess;
+    update_tiles_kernel<WT, 2, COMMIT><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+  } else {
+    if (a.n_index == 0) return cudaSuccess;
+    const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
+    update_index_kernel<WT, COMMIT><<<(unsigned)blocks, kThreads, 0, s>>>(a);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_update(int kind, int dtype, const UpdateArgs &a, cudaStream_t s, int) {
+  if (dtype == COPES_BF16)
+    return a.fuse_commit ? launch_update_typed<__nv_bfloat16, true>(kind, a, s)
+                         : launch_update_typed<__nv_bfloat16, false>(kind, a, s);
+  return a.fuse_commit ? launch_update_typed<float, true>(kind, a, s)
+                       : launch_update_typed<float, false>(kind, a, s);
+}
+
+// -------------------------------------------------------------------------- debug
+__global__ void debug_philox_kernel(uint64_t seed, uint64_t q0, uint64_t n, uint32_t aux,
+                                    uint32_t tag, uint32_t *out) {
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const uint64_t q = q0 + i;
+  uint32_t x[4];
+  philox4x32_10((uint32_t)q, (uint32_t)(q >> 32), aux, tag, (uint32_t)seed,
+                (uint32_t)(seed >> 32), x);
+  reinterpret_cast<uint4 *>(out)[i] = make_uint4(x[0], x[1], x[2], x[3]);
+}
+
+__global__ void debug_normals_kernel(uint64_t seed, uint32_t tag, uint64_t g0, uint64_t n,
+                                     float *out) {
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  out[i] = index_noise(g0 + i, tag, (uint32_t)seed, (uint32_t)(seed >> 32));
+}
+
+__global__ void debug_transform_kernel(const uint32_t *words, uint64_t n, float *out) {
+  const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < n) out[i] = normal_from_word(words[i]);
+}
+
+static unsigned blocks_for(uint64_t n) { return (unsigned)((n + kThreads - 1) / kThreads); }
+
+cudaError_t launch_debug_philox(uint64_t seed, uint64_t q0, uint64_t n, uint32_t aux,
+                                uint32_t tag, uint32_t *out, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  debug_philox_kernel<<<blocks_for(n), kThreads, 0, s>>>(seed, q0, n, aux, tag, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_debug_normals(uint64_t seed, uint32_t tag, uint64_t g0, uint64_t n,
+                                 float *out, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  debug_normals_kernel<<<blocks_for(n), kThreads, 0, s>>>(seed, tag, g0, n, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_debug_transform(const uint32_t *words, uint64_t n, float *out,
+                                   cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  debug_transform_kernel<<<blocks_for(n), kThreads, 0, s>>>(words, n, out);
+  return cudaGetLastError();
+}
+
+unsigned read_and_clear_es_errors() {
+  unsigned v = 0, zero = 0;
+  cudaMemcpyFromSymbol(&v, g_es_error, sizeof(v));
+  if (v) cudaMemcpyToSymbol(g_es_error, &zero, sizeof(zero));
+  return v;
+}
+
+}  // namespace copes

@@ -1,0 +1,221 @@
+// Partition kernels (Eq. 7; Algorithm 1 "sample a partition"; Supp. A.8 partition
+// replay): the hash partition's per-tile histogram, per-bucket exclusive scan and
+// order-preserving scatter into sorted int64 lists, and the random-chunk map.
+#include "copes_internal.h"
+
+namespace copes {
+
+__device__ unsigned int g_partition_error = 0;
+
+constexpr int kPartThreads = 256;
+constexpr int kPartWarps = kPartThreads / 32;
+
+__device__ __forceinline__ uint32_t hash_bucket(uint64_t e, uint32_t tensor_id, uint32_t k0,
+                                                uint32_t k1, int K) {
+  uint32_t x[4];
+  const uint64_t q = e >> 2;
+  philox4x32_10((uint32_t)q, (uint32_t)(q >> 32), tensor_id, COPES_TAG_PARTITION, k0, k1, x);
+  const uint32_t s = (uint32_t)e & 3u;
+  const uint32_t w = s == 0 ? x[0] : (s == 1 ? x[1] : (s == 2 ? x[2] : x[3]));
+  return (uint32_t)(((uint64_t)w * (uint64_t)K) >> 32);
+}
+
+// The tensor owning hash tile `tile`: the last entry with tile_begin <= tile (the host
+// table lists only tensors with at least one element).
+__device__ int owner_tensor(const HashTensor *tensors, int n_tensors, uint64_t tile) {
+  int lo = 0, hi = n_tensors - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (tensors[mid].tile_begin <= tile) lo = mid;
+    else hi = mid - 1;
+  }
+  return lo;
+}
+
+__global__ void __launch_bounds__(kPartThreads) hash_hist_kernel(
+    const HashTensor *tensors, int n_tensors, int K, uint64_t seed, uint32_t *hist,
+    unsigned long long *totals) {
+  __shared__ uint32_t s_h[COPES_MAX_K];
+  __shared__ int s_t;
+  const uint64_t tile = blockIdx.x;
+  if (threadIdx.x == 0) s_t = owner_tensor(tensors, n_tensors, tile);
+  for (int k = threadIdx.x; k < K; k += kPartThreads) s_h[k] = 0;
+  __syncthreads();
+  const HashTensor T = tensors[s_t];
+  const uint64_t e0 = (tile - T.tile_begin) * kHashTile;
+  const uint64_t e1 = min(e0 + kHashTile, T.numel);
+  const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+  for (uint64_t e = e0 + 4ull * threadIdx.x; e < e1; e += 4ull * kPartThreads) {
+    uint32_t x[4];
+    const uint64_t q = e >> 2;  // e is a multiple of 4: tiles start at multiples of 16384
+    philox4x32_10((uint32_t)q, (uint32_t)(q >> 32), T.tensor_id, COPES_TAG_PARTITION, k0, k1, x);
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (e + k < e1) atomicAdd(&s_h[(uint32_t)(((uint64_t)x[k] * (uint64_t)K) >> 32)], 1u);
+  }
+  __syncthreads();
+  for (int k = threadIdx.x; k < K; k += kPartThreads) {
+    hist[tile * K + k] = s_h[k];
+    if (s_h[k]) atomicAdd(&totals[k], (unsigned long long)s_h[k]);
+  }
+}
+
+// Block k: exclusive prefix sum over tiles of hist[tile][k] -> offsets[tile][k].
+__global__ void __launch_bounds__(1024) hash_scan_kernel(const uint32_t *hist, uint64_t n_htiles,
+                                                         int K, uint64_t *offsets) {
+  __shared__ unsigned long long s_part[1024];
+  const int k = blockIdx.x;
+  const uint64_t per = (n_htiles + 1023) / 1024;
+  const uint64_t t0 = min((uint64_t)threadIdx.x * per, n_htiles);
+  const uint64_t t1 = min(t0 + per, n_htiles);
+  unsigned long long sum = 0;
+  for (uint64_t t = t0; t < t1; ++t) sum += hist[t * K + k];
+  s_part[threadIdx.x] = sum;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long acc = 0;
+    for (int i = 0; i < 1024; ++i) {
+      const unsigned long long v = s_part[i];
+      s_part[i] = acc;
+      acc += v;
+    }
+  }
+  __syncthreads();
+  unsigned long long acc = s_part[threadIdx.x];
+  for (uint64_t t = t0; t < t1; ++t) {
+    offsets[t * K + k] = acc;
+    acc += hist[t * K + k];
+  }
+}
+
+struct ListTable {
+  int64_t *list[COPES_MAX_K];
+};
+
+// One block per hash tile; 256 consecutive elements per step, in element order, so the
+// lists come out sorted.  Within a step an element's position is its bucket's running
+// offset + the counts of earlier warps + its rank among equal buckets of its warp.
+__global__ void __launch_bounds__(kPartThreads) hash_scatter_kernel(
+    const HashTensor *tensors, int n_tensors, int K, uint64_t seed, const uint64_t *offsets,
+    const ListTable lists) {
+  __shared__ unsigned long long s_run[COPES_MAX_K];
+  __shared__ uint32_t s_tot[COPES_MAX_K];
+  __shared__ uint32_t s_wc[kPartWarps][COPES_MAX_K];
+  __shared__ int s_t;
+  const uint64_t tile = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) s_t = owner_tensor(tensors, n_tensors, tile);
+  for (int k = threadIdx.x; k < K; k += kPartThreads) s_run[k] = offsets[tile * K + k];
+  __syncthreads();
+  const HashTensor T = tensors[s_t];
+  const uint64_t e0 = (tile - T.tile_begin) * kHashTile;
+  const uint64_t e1 = min(e0 + kHashTile, T.numel);
+  const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+  const unsigned lt_mask = (1u << lane) - 1u;
+  for (uint64_t step = e0; step < e1; step += kPartThreads) {
+    const uint64_t e = step + threadIdx.x;
+    const bool valid = e < e1;
+    const uint32_t b = valid ? hash_bucket(e, T.tensor_id, k0, k1, K) : 0xFFFFFFFFu;
+    for (int k = lane; k < K; k += 32) s_wc[warp][k] = 0;
+    __syncwarp();
+    const unsigned peers = __match_any_sync(0xffffffffu, b);
+    const int rank = __popc(peers & lt_mask);
+    if (valid && (__ffs(peers) - 1) == lane) s_wc[warp][b] = (uint32_t)__popc(peers);
+    __syncthreads();
+    for (int k = threadIdx.x; k < K; k += kPartThreads) {
+      uint32_t acc = 0;
+      for (int w = 0; w < kPartWarps; ++w) {
+        const uint32_t c = s_wc[w][k];
+        s_wc[w][k] = acc;
+        acc += c;
+      }
+      s_tot[k] = acc;
+    }
+    __syncthreads();
+    if (valid) lists.list[b][s_run[b] + s_wc[warp][b] + (uint32_t)rank] = (int64_t)(T.offset + e);
+    __syncthreads();
+    for (int k = threadIdx.x; k < K; k += kPartThreads) s_run[k] += s_tot[k];
+    __syncthreads();
+  }
+}
+
+// Random chunk map: chunk c has key = word 0 of Philox(seed; c, 0, CHUNK tag); its rank
+// under (key, c) order is counted against every other chunk; map[c] = rank K / n.
+__global__ void __launch_bounds__(kPartThreads) chunk_rank_kernel(uint64_t n, int K, uint64_t seed,
+                                                                  uint32_t *map) {
+  __shared__ uint32_t s_key[1024];
+  const uint64_t c = (uint64_t)blockIdx.x * kPartThreads + threadIdx.x;
+  const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+  uint32_t mine = 0;
+  if (c < n) {
+    uint32_t x[4];
+    philox4x32_10((uint32_t)c, (uint32_t)(c >> 32), 0u, COPES_TAG_CHUNK, k0, k1, x);
+    mine = x[0];
+  }
+  uint64_t less = 0;
+  for (uint64_t base = 0; base < n; base += 1024) {
+    for (int i = threadIdx.x; i < 1024; i += kPartThreads) {
+      const uint64_t cc = base + i;
+      uint32_t key = 0xFFFFFFFFu;
+      if (cc < n) {
+        uint32_t x[4];
+        philox4x32_10((uint32_t)cc, (uint32_t)(cc >> 32), 0u, COPES_TAG_CHUNK, k0, k1, x);
+        key = x[0];
+      }
+      s_key[i] = key;
+    }
+    __syncthreads();
+    if (c < n) {
+      const int m = (int)min((uint64_t)1024, n - base);
+      for (int i = 0; i < m; ++i) {
+        const uint32_t key = s_key[i];
+        less += (key < mine) || (key == mine && base + i < c);
+      }
+    }
+    __syncthreads();
+  }
+  if (c < n) map[c] = (uint32_t)((less * (uint64_t)K) / n);
+}
+
+cudaError_t launch_hash_hist(const HashTensor *tensors, int n_tensors, uint64_t n_htiles, int K,
+                             uint64_t seed, uint32_t *hist, unsigned long long *totals,
+                             cudaStream_t s) {
+  if (n_htiles == 0) return cudaSuccess;
+  hash_hist_kernel<<<(unsigned)n_htiles, kPartThreads, 0, s>>>(tensors, n_tensors, K, seed, hist,
+                                                                totals);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_hash_scan(const uint32_t *hist, uint64_t n_htiles, int K, uint64_t *offsets,
+                             cudaStream_t s) {
+  if (n_htiles == 0) return cudaSuccess;
+  hash_scan_kernel<<<K, 1024, 0, s>>>(hist, n_htiles, K, offsets);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_hash_scatter(const HashTensor *tensors, int n_tensors, uint64_t n_htiles,
+                                int K, uint64_t seed, const uint64_t *offsets,
+                                int64_t *const *lists, cudaStream_t s) {
+  if (n_htiles == 0) return cudaSuccess;
+  ListTable t;
+  for (int k = 0; k < COPES_MAX_K; ++k) t.list[k] = k < K ? lists[k] : nullptr;
+  hash_scatter_kernel<<<(unsigned)n_htiles, kPartThreads, 0, s>>>(tensors, n_tensors, K, seed,
+                                                                   offsets, t);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,
+                                    cudaStream_t s) {
+  const unsigned blocks = (unsigned)((n_chunks + kPartThreads - 1) / kPartThreads);
+  chunk_rank_kernel<<<blocks, kPartThreads, 0, s>>>(n_chunks, K, seed, map);
+  return cudaGetLastError();
+}
+
+unsigned read_and_clear_partition_errors() {
+  unsigned v = 0, zero = 0;
+  cudaMemcpyFromSymbol(&v, g_partition_error, sizeof(v));
+  if (v) cudaMemcpyToSymbol(g_partition_error, &zero, sizeof(zero));
+  return v;
+}
+
+}  // namespace copes

@@ -1,0 +1,122 @@
+"""Host-side schedules of the CoPES ES core (orchestration only; every step is a library
+kernel launched through the ``copes`` binding).
+
+round_robin_visit  one ES iteration on one subspace: N perturbed evaluations, restore,
+                   shaping, fused update + context commit (the cooperative-coevolution
+                   visit; one "cycle" visits k = 0 .. K-1 in order).
+sync_step          one CoPES training step (Algorithm 1): every subspace's N_k = N / K
+                   members are evaluated under the same pre-update context, rewards are
+                   standardised jointly (Eq. 12) or per subspace (Sec. 4.4 ablation), and
+                   all K subspace updates are composed (Eq. 13) before the commit.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+from typing import Callable, List, Optional, Sequence
+
+import numpy as np
+import torch
+
+from . import copes
+
+
+@dataclass
+class ESConfig:
+    n_members: int
+    sigma: float
+    alpha: float
+    shaping: str = "zscore"
+    pairing: int = copes.ANTITHETIC
+    convention: int = copes.COEF_OPENAI
+    dimension_aware: bool = False
+    base_seed: int = 33
+
+
+def sigma_k(cfg: ESConfig, d: int, d_k: int) -> float:
+    """Eq. 11 when dimension-aware, else the configured sigma."""
+    return copes.sigma_eff(cfg.sigma, d, d_k, cfg.dimension_aware)
+
+
+def round_robin_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iteration: int,
+                      cfg: ESConfig, d: int, rewards: torch.Tensor,
+                      evaluate: Optional[Callable[[int], None]] = None,
+                      fitness_out: Optional[torch.Tensor] = None,
+                      events: Optional[dict] = None) -> torch.Tensor:
+    """One ES iteration on subspace k.  `rewards` (device fp32 [N]) holds the members'
+    rewards; `evaluate(i)` runs while member i's perturbation is live (it may write
+    rewards[i]).  Returns the shaped fitness."""
+    nid, sign, P = copes.member_table(cfg.n_members, cfg.pairing)
+    seeds = copes.member_seeds(cfg.base_seed, iteration, k, P)
+    s_k = sigma_k(cfg, d, sub.numel)
+    for i in range(cfg.n_members):
+        _timed(events, "perturb", lambda: copes.perturb(arena, sub, int(seeds[nid[i]]), float(sign[i]) * s_k))
+        if evaluate is not None:
+            evaluate(i)
+    _timed(events, "restore", lambda: copes.restore(arena, sub))
+    f = fitness_out if fitness_out is not None else torch.empty_like(rewards)
+    _timed(events, "shape", lambda: copes.shape_fitness(rewards, cfg.shaping, out=f))
+    coef = copes.step_coef(cfg.alpha, cfg.n_members, s_k, cfg.convention)
+    _timed(events, "update", lambda: copes.update(arena, sub, nid, sign, f, seeds, coef, fuse_commit=True))
+    return f
+
+
+def sync_step(arena: copes.Arena, subs: Sequence[copes.SubspaceHandle], iteration: int,
+              cfg: ESConfig, d: int, rewards: torch.Tensor,
+              evaluate: Optional[Callable[[int, int], None]] = None,
+              joint: bool = True) -> torch.Tensor:
+    """Algorithm 1: N = cfg.n_members split into N_k = N / K per subspace; rewards is the
+    device fp32 [N] vector laid out subspace by subspace (member i of subspace k at
+    k N_k + i).  evaluate(k, i) runs while that member's perturbation is live."""
+    K = len(subs)
+    if cfg.n_members % K:
+        raise ValueError("N must be divisible by K (Sec. 3.2)")
+    n_k = cfg.n_members // K
+    nid, sign, P = copes.member_table(n_k, cfg.pairing)
+    seeds = [copes.member_seeds(cfg.base_seed, iteration, k, P) for k in range(K)]
+    for k, sub in enumerate(subs):
+        s_k = sigma_k(cfg, d, sub.numel)
+        for i in range(n_k):
+            copes.perturb(arena, sub, int(seeds[k][nid[i]]), float(sign[i]) * s_k)
+            if evaluate is not None:
+                evaluate(k, i)
+        copes.restore(arena, sub)  # the next subspace is evaluated under the same context
+    if joint:
+        f = copes.shape_fitness(rewards, copes.SHAPE_ZSCORE if cfg.shaping == "zscore" else cfg.shaping)
+    else:
+        group = torch.arange(cfg.n_members, device=rewards.device, dtype=torch.int32) // n_k
+        f = copes.shape_fitness(rewards, copes.SHAPE_ZSCORE_GROUPED, group=group)
+    for k, sub in enumerate(subs):  # every g_k from the same pre-update theta (disjoint supports)
+        s_k = sigma_k(cfg, d, sub.numel)
+        coef = copes.step_coef(cfg.alpha, n_k, s_k, cfg.convention)
+        copes.update(arena, sub, nid, sign, f[k * n_k:(k + 1) * n_k], seeds[k], coef, fuse_commit=True)
+    return f
+
+
+def _timed(events: Optional[dict], name: str, fn):
+    if events is None:
+        return fn()
+    start = torch.cuda.Event(enable_timing=True)
+    end = torch.cuda.Event(enable_timing=True)
+    start.record()
+    out = fn()
+    end.record()
+    events.setdefault(name, []).append((start, end))
+    return out
+
+
+def build_subspaces(layout: copes.Layout, mode: str, K: int, group_of: Optional[List[int]] = None,
+                    seed: int = 0, chunk: int = 65536, tile_size: int = copes.DEFAULT_TILE):
+    """All K subspaces of a partition (tiles for range modes, index lists for hash)."""
+    if mode == "hash":
+        return copes.hash_partition(layout, K, seed)
+    if mode == "contiguous":
+        return [copes.subspace_build(layout, copes.PART_CONTIGUOUS, K, k, tile_size=tile_size) for k in range(K)]
+    if mode == "groups":
+        return [copes.subspace_build(layout, copes.PART_TENSOR_GROUPS, K, k, group_of=group_of,
+                                     tile_size=tile_size) for k in range(K)]
+    if mode == "random_chunks":
+        n_chunks = (layout.d_pad + chunk - 1) // chunk
+        cmap = copes.random_chunk_map(n_chunks, K, seed)
+        return [copes.subspace_build(layout, copes.PART_RANDOM_CHUNKS, K, k, seed=seed, chunk=chunk,
+                                     chunk_map=cmap, tile_size=tile_size) for k in range(K)]
+    raise ValueError(mode)

@@ -1,0 +1,141 @@
+"""The C ABI library without a GPU: it loads, exports every function include/copes.h
+declares, its host-side logic matches the oracle, and invalid arguments come back as
+error codes before any CUDA call."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_02391_gb300 import build, copes
+    if not os.path.exists(copes.LIB_PATH):
+        try:
+            build.build()
+        except RuntimeError as e:
+            pytest.skip(f"cannot build libcopes.so here: {e}")
+    return copes.load()
+
+
+def declared_functions():
+    text = open(os.path.join(ROOT, "include", "copes.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(copes_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 20
+    for name in names:
+        assert hasattr(lib, name), name
+    from paper_2608_02391_gb300 import copes
+    assert set(names) == set(copes.SIGNATURES)
+
+
+def test_version_and_error_strings(lib):
+    assert b"sm_103a" in lib.copes_version()
+    assert lib.copes_perturb(None, None, 0, 1.0, None) == -1
+    buf = ctypes.create_string_buffer(256)
+    n = lib.copes_last_error(buf, 256)
+    assert n > 0 and b"copes_perturb" in buf.value
+
+
+def test_host_helpers_match_oracle(lib):
+    from paper_2608_02391_gb300 import copes
+    for args in [(33, 0, 0, 0), (33, 5, 7, 63), (2**63 + 11, 2**31, 3, 1)]:
+        assert copes.member_seed(*args) == oracle.member_seed(*args)
+    for n, pairing in [(8, copes.ANTITHETIC), (128, copes.ANTITHETIC), (5, copes.ONE_SIDED)]:
+        a = copes.member_table(n, pairing)
+        b = oracle.member_table(n, pairing)
+        assert np.array_equal(a[0], b[0]) and np.array_equal(a[1], b[1]) and a[2] == b[2]
+    assert copes.sigma_eff(1e-3, 4e9, 1e9) == oracle.sigma_eff(1e-3, 4e9, 1e9)
+    for conv in (copes.COEF_PAPER, copes.COEF_OPENAI):
+        assert copes.step_coef(5e-4, 32, 1e-3, conv) == oracle.step_coef(5e-4, 32, 1e-3, conv)
+    numel = [1000, 64, 7, 4096, 130, 1, 2500]
+    assert np.array_equal(copes.Layout(numel).offsets, oracle.layout(numel))
+
+
+def _expected_tiles(ranges, tile):
+    out = []
+    for b, e in ranges:
+        for s in range(b, e, tile):
+            out.append((s, min(s + tile, e)))
+    return out
+
+
+def test_subspace_build_tile_counts_match_oracle_ranges(lib):
+    from paper_2608_02391_gb300 import copes
+    numel = [1000, 64, 7, 4096, 130, 1, 2500]
+    L = copes.Layout(numel)
+    count = ctypes.c_uint64()
+    for K in (1, 3, 4):
+        for k in range(K):
+            spec = copes.PartitionSpec(copes.PART_CONTIGUOUS, K, 0, 0, None)
+            rc = lib.copes_subspace_build(ctypes.byref(L.desc), ctypes.byref(spec), k, 100, None, None, 0,
+                                          ctypes.byref(count), None)
+            assert rc == 0
+            assert count.value == len(_expected_tiles(oracle.contiguous_ranges(numel, K, k), 100))
+    groups = np.array([0, 1, 1, 0, 2, 2, 1], np.int32)
+    for k in range(3):
+        spec = copes.PartitionSpec(copes.PART_TENSOR_GROUPS, 3, 0, 0, groups.ctypes.data_as(ctypes.c_void_p))
+        assert lib.copes_subspace_build(ctypes.byref(L.desc), ctypes.byref(spec), k, 512, None, None, 0,
+                                        ctypes.byref(count), None) == 0
+        assert count.value == len(_expected_tiles(oracle.group_ranges(numel, groups, k), 512))
+
+
+def test_invalid_arguments_are_rejected_before_any_launch(lib):
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    p = copes.Params(fake, fake + 3, 100, copes.BF16)  # misaligned master
+    s = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
+    assert lib.copes_perturb(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, None) == copes.ERR_ALIGNMENT
+    p = copes.Params(fake, fake, 100, 7)
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
+    p = copes.Params(fake, fake, 100, copes.BF16)
+    bad = copes.Subspace(9, None, 0, None, 0)
+    assert lib.copes_context_commit(ctypes.byref(p), ctypes.byref(bad), None) == copes.ERR_INVALID_ARG
+    idx = copes.Subspace(copes.SUBSPACE_INDICES, None, 0, fake + 8, 10)
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(idx), None) == copes.ERR_ALIGNMENT
+    assert lib.copes_perturb(ctypes.byref(p), ctypes.byref(s), 1, float("nan"), None) == copes.ERR_INVALID_ARG
+    assert lib.copes_shape_fitness(fake, 0, None, copes.SHAPE_ZSCORE, fake, None) == copes.ERR_SIZE
+    assert lib.copes_shape_fitness(fake, 300, None, copes.SHAPE_ZSCORE, fake, None) == copes.ERR_SIZE
+    assert lib.copes_shape_fitness(fake, 8, None, copes.SHAPE_ZSCORE_GROUPED, fake, None) == copes.ERR_INVALID_ARG
+    nid = np.array([0, 0, 1, 5], np.int32)
+    sg = np.array([1, -1, 1, -1], np.int8)
+    seeds = np.zeros(2, np.uint64)
+    P = ctypes.c_void_p
+    assert lib.copes_update(ctypes.byref(p), ctypes.byref(s), 4, nid.ctypes.data_as(P), sg.ctypes.data_as(P),
+                            fake, 2, seeds.ctypes.data_as(P), 0.1, 1, None) == copes.ERR_INVALID_ARG
+    nid[3] = 1
+    sg[3] = 0
+    assert lib.copes_update(ctypes.byref(p), ctypes.byref(s), 4, nid.ctypes.data_as(P), sg.ctypes.data_as(P),
+                            fake, 2, seeds.ctypes.data_as(P), 0.1, 1, None) == copes.ERR_INVALID_ARG
+    assert lib.copes_update(ctypes.byref(p), ctypes.byref(s), 300, nid.ctypes.data_as(P), sg.ctypes.data_as(P),
+                            fake, 2, seeds.ctypes.data_as(P), 0.1, 1, None) == copes.ERR_SIZE
+    L = copes.Layout([1000, 2000])
+    need = lib.copes_hash_workspace_bytes(ctypes.byref(L.desc), 16)
+    assert need > 0
+    counts = np.zeros(16, np.uint64)
+    assert lib.copes_hash_count(ctypes.byref(L.desc), 16, 1, fake, need - 16, counts.ctypes.data_as(P),
+                                None) == copes.ERR_WORKSPACE
+    assert lib.copes_hash_count(ctypes.byref(L.desc), 65, 1, fake, need, counts.ctypes.data_as(P),
+                                None) == copes.ERR_INVALID_ARG
+    assert lib.copes_random_chunk_map(0, 4, 1, fake, None) == copes.ERR_SIZE
+    assert lib.copes_random_chunk_map((1 << 20) + 1, 4, 1, fake, None) == copes.ERR_SIZE
+    spec = copes.PartitionSpec(copes.PART_HASH, 4, 0, 0, None)
+    cnt = ctypes.c_uint64()
+    assert lib.copes_subspace_build(ctypes.byref(L.desc), ctypes.byref(spec), 0, 100, None, None, 0,
+                                    ctypes.byref(cnt), None) == copes.ERR_INVALID_ARG
+    spec = copes.PartitionSpec(copes.PART_CONTIGUOUS, 4, 0, 0, None)
+    assert lib.copes_subspace_build(ctypes.byref(L.desc), ctypes.byref(spec), 4, 100, None, None, 0,
+                                    ctypes.byref(cnt), None) == copes.ERR_INVALID_ARG
+    assert lib.copes_subspace_build(ctypes.byref(L.desc), ctypes.byref(spec), 0, 0, None, None, 0,
+                                    ctypes.byref(cnt), None) == copes.ERR_SIZE
+    assert lib.copes_member_table(7, copes.ANTITHETIC, fake, fake) == copes.ERR_INVALID_ARG
