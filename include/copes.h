@@ -219,6 +219,25 @@ int copes_hash_count(const copes_layout_desc *layout, int K, uint64_t seed, void
 int copes_hash_fill(const copes_layout_desc *layout, int K, uint64_t seed, void *workspace,
                     size_t workspace_bytes, int64_t *const *lists, cudaStream_t stream);
 
+/* Hash partition for callers that cannot allocate device memory -- for instance an ES
+ * trainer sharing the GPU with a rollout engine that reserved nearly all free HBM for its
+ * KV cache, or code inside a framework that owns the memory pool and forbids cudaMalloc.
+ * (The paper has no counterpart: this is a deployment variant of copes_hash_count +
+ * copes_hash_fill.)  Same partition and same output as those two calls, but the scratch
+ * is a fixed 8 MiB array inside the library, held by every GPU that loads it until the
+ * process exits; nothing is allocated on the device or the host.
+ *  - lists == NULL: counts every subspace into counts[K] (host) and SYNCHRONISES stream.
+ *  - otherwise also writes the sorted lists: lists[k] (device, capacity[k] int64, host
+ *    arrays of K) must hold counts[k] entries, else COPES_ERR_WORKSPACE and no list is
+ *    written; the fill is asynchronous on stream.
+ * A layout whose scratch exceeds 8 MiB (about 12 K bytes per 16,384-element tile) is
+ * rejected with COPES_ERR_SIZE.  The first call on a device looks up the array's device
+ * address with that device current; make that first call before any stream capture.
+ * Every call reuses the same array, so calls whose GPU work overlaps race: serialise them. */
+int copes_hash_partition_static(const copes_layout_desc *layout, int K, uint64_t seed,
+                                int64_t *const *lists, const uint64_t *capacity,
+                                uint64_t *counts, cudaStream_t stream);
+
 /* ------------------------------------------------------------------------- ES steps */
 
 /* Perturb (Eq. 8, Algorithm 1 "set theta_{k,i}"): for every g in S,

@@ -80,6 +80,7 @@ SIGNATURES = {
     "copes_hash_workspace_bytes": (_SZ, [_VP, _I32]),
     "copes_hash_count": (_I32, [_VP, _I32, _U64, _VP, _SZ, _VP, _VP]),
     "copes_hash_fill": (_I32, [_VP, _I32, _U64, _VP, _SZ, _VP, _VP]),
+    "copes_hash_partition_static": (_I32, [_VP, _I32, _U64, _VP, _VP, _VP, _VP]),
     "copes_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
     "copes_restore": (_I32, [_VP, _VP, _VP]),
     "copes_context_commit": (_I32, [_VP, _VP, _VP]),
@@ -273,6 +274,21 @@ def hash_partition(layout: Layout, K: int, seed: int, device="cuda", stream=None
     _check(L.copes_hash_fill(ctypes.byref(layout.desc), K, seed, _ptr(ws), nbytes, ptrs, s))
     if stream is not None:
         ws.record_stream(stream)  # freed in stream order with the fill's kernels
+    return [SubspaceHandle(SUBSPACE_INDICES, t[:int(c)], int(c)) for t, c in zip(lists, counts)]
+
+
+def hash_partition_static(layout: Layout, K: int, seed: int, device="cuda", stream=None) -> List[SubspaceHandle]:
+    """copes_hash_partition_static: the same K sorted index lists as hash_partition, built
+    on the library's fixed static scratch instead of a workspace (for callers that cannot
+    allocate device scratch; the lists themselves are still allocated here by torch)."""
+    L, s = load(), _stream(stream)
+    counts = np.zeros(K, np.uint64)
+    _check(L.copes_hash_partition_static(ctypes.byref(layout.desc), K, seed, None, None, _np_ptr(counts), s))
+    lists = [torch.empty(max(int(c), 2), dtype=torch.int64, device=device) for c in counts]
+    ptrs = (ctypes.c_void_p * K)(*[t.data_ptr() for t in lists])
+    caps = np.array([t.numel() for t in lists], np.uint64)
+    _check(L.copes_hash_partition_static(ctypes.byref(layout.desc), K, seed, ptrs, _np_ptr(caps),
+                                         _np_ptr(counts), s))
     return [SubspaceHandle(SUBSPACE_INDICES, t[:int(c)], int(c)) for t, c in zip(lists, counts)]
 
 

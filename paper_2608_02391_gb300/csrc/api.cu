@@ -149,6 +149,8 @@ int emit_tiles(const Ranges &r, uint64_t tile_size, uint64_t *tiles, uint64_t ca
 
 }  // namespace
 
+void copes::set_last_error(const char *message) { g_message = message; }
+
 extern "C" {
 
 const char *copes_version(void) { return "copes-gb300 0.1 (sm_103a)"; }

@@ -121,6 +121,9 @@ cudaError_t launch_hash_scatter(const HashTensor *tensors, int n_tensors, uint64
 cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,
                                     cudaStream_t s);
 
+// Sets the calling thread's message reported by copes_last_error.
+void set_last_error(const char *message);
+
 // Device error words of each translation unit: read and clear (synchronous).
 unsigned read_and_clear_es_errors();
 unsigned read_and_clear_partition_errors();
