@@ -54,6 +54,8 @@ def parse():
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice"],
+                    help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling")
     return ap.parse_args()
 
 
@@ -184,6 +186,10 @@ def run_reference(args, wl):
 
 
 def workload_config(wl, args):
+    if wl.name != "4b":
+        return {"workload": f"{wl.name}: {wl.d} parameters in {len(wl.tensors)} tensors, K={wl.K}, "
+                            f"N={wl.n_members} antithetic (profiling case)", "params": wl.d, "K": wl.K,
+                "N": wl.n_members, "tile": args.tile}
     return {"workload": "4B decoder-shaped bf16 set, fp32 master, K=8 layer blocks, N=32 antithetic",
             "params": wl.d, "layers": 36, "hidden": 2560, "mlp": 9728, "vocab": 151936, "tied": True,
             "K": wl.K, "N": wl.n_members, "sigma": wl.sigma, "alpha": wl.alpha, "shaping": wl.shaping,
@@ -194,7 +200,7 @@ def workload_config(wl, args):
 def main():
     args = parse()
     from paper_2608_02391_gb300 import workloads
-    wl = workloads.workload("4b")
+    wl = workloads.workload(args.case)
     if args.impl == "reference":
         return run_reference(args, wl)
 

@@ -15,7 +15,7 @@
  *    (copes_layout).  The caller allocates two flat device buffers over that space: the
  *    working weights w (bf16 or fp32; what the model reads) and the fp32 master theta.
  *  - Noise: eps_seed[g] is a standard normal that depends only on (seed, g).  It is
- *    Phi^-1(u) of the odd 24-bit uniform u = ((x >> 8) | 1) * 2^-24, where x is word
+ *    Phi^-1(u) of the odd-lattice uniform u = ((x & 0x7FFFFE) | 1) * 2^-23, where x is word
  *    (g & 3) of Philox4x32-10 (Salmon et al., SC'11) at counter (lo32(g >> 2),
  *    hi32(g >> 2), 0, 0) under key (lo32(seed), hi32(seed)).
  *  - Ownership: the caller owns every device buffer (weights, masters, rewards,

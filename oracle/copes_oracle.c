@@ -18,7 +18,7 @@
  *     perturbation is its seed, and its noise is regenerated from (seed, index).
  *   - Gaussian directions eps ~ N(0, I): Eq. 3 and Eq. 8.  The transform from a Philox
  *     word to a normal is this project's choice (the paper is silent): the exact
- *     standard-normal quantile of a 24-bit odd uniform.
+ *     standard-normal quantile of an odd 23-bit-lattice uniform.
  *   - Perturbation theta + sigma_k * P_k eps: Eq. 8 (Sec. 3.2); antithetic signs +/-.
  *   - Dimension-aware scale sigma_k = sigma * sqrt(d / d_k): Eq. 11.
  *   - Restore / context commit from the fp32 master: Sec. 3.3 weight backup, Supp. A.8
@@ -104,10 +104,11 @@ void oracle_philox_stream(uint64_t seed, uint64_t q0, uint64_t n, uint32_t aux, 
 
 /* ------------------------------------------------------------------------------------
  * Uniform and normal.
- * u(x) = ((x >> 8) | 1) * 2^-24: an odd multiple of 2^-24, strictly inside (0, 1), so
- * the quantile below is finite.  u and 1 - u are both exact in fp32 and fp64.
+ * u(x) = ((x & 0x7FFFFE) | 1) * 2^-23: bits 1..22 of the word, made odd -- an odd
+ * multiple of 2^-23, strictly inside (0, 1), so the quantile below is finite.  u and
+ * 1 - u are both exact in fp32 and fp64, and the lattice is symmetric about 1/2.
  * ------------------------------------------------------------------------------------ */
-double oracle_uniform(uint32_t x) { return ldexp((double)((x >> 8) | 1u), -24); }
+double oracle_uniform(uint32_t x) { return ldexp((double)((x & 0x7FFFFEu) | 1u), -23); }
 
 /* Standard-normal quantile Phi^-1(u), solved by Newton's method on the definition
  * Phi(x) = erfc(-x / sqrt 2) / 2, using libm's erf / erfc.

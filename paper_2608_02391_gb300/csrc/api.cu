@@ -13,6 +13,7 @@
 #include <vector>
 
 #include "copes_internal.h"
+#include "normal_coeffs.h"
 
 using copes::ElemArgs;
 using copes::UpdateArgs;
@@ -119,6 +120,12 @@ int run_elementwise(int op, const copes_params *p, const copes_subspace *S, uint
   a.tag = tag;
   a.a = a_val;
   a.b = b_val;
+  // the scale folded into the normal's polynomial: a * eps = x * (a * R(L))
+  static const float central[] = COPES_NORMAL_CENTRAL_COEFFS;
+  static const float tail[] = COPES_NORMAL_TAIL_COEFFS;
+  for (int i = 0; i <= COPES_NORMAL_CENTRAL_DEGREE; ++i) a.coeffs.central[i] = a_val * central[i];
+  for (int i = 0; i <= COPES_NORMAL_TAIL_DEGREE; ++i) a.coeffs.tail[i] = a_val * tail[i];
+  copes::philox_round_keys(a.seed_lo, a.seed_hi, a.rk);
   return launch_status(copes::launch_elementwise(op, S->kind, p->dtype, a, s), who);
 }
 

@@ -23,33 +23,85 @@ __device__ __forceinline__ float sqrt_approx(float x) {
 
 template <int N>
 __device__ __forceinline__ float horner(const float (&c)[N], float v) {
+  // Horner's rule, highest coefficient first
   float r = c[N - 1];
 #pragma unroll
-  for (int i = N - 2; i >= 0; --i) r = fmaf(r, v, c[i]);
+  for (int i = N - 2; i >= 0; --i) r = __fmaf_rn(r, v, c[i]);
   return r;
 }
 
-// Standard normal from one Philox word: eps = Phi^-1(u), u = ((w >> 8) | 1) * 2^-24.
-// x = 2u - 1 is formed exactly from the float with exponent 1 and mantissa w >> 9
-// (value 2 + (w >> 9) 2^-22):  x = (that - 3) + 2^-23, both steps exact.  Then
-// eps = sqrt(2) erfinv(x) = x * R(L), L = log2(1 - x^2), with R a fitted polynomial in L
-// on the central range and in sqrt(-L) on the tail (coefficients: normal_coeffs.h).
-// R is evaluated relative to its own value, so eps has a small relative error for all x,
-// including x near 0 (where L -> 0) and near +-1.
-__device__ __forceinline__ float normal_from_word(uint32_t w) {
-  const float f = __uint_as_float((w >> 9) | 0x40000000u);
-  const float x = __fadd_rn(__fadd_rn(f, -3.0f), 0x1p-23f);
-  const float t = __fmaf_rn(-x, x, 1.0f);
-  const float L = lg2_approx(t);
-  float r;
-  if (__builtin_expect(L >= COPES_NORMAL_L_SPLIT, 1)) {
-    constexpr float c[COPES_NORMAL_CENTRAL_DEGREE + 1] = COPES_NORMAL_CENTRAL_COEFFS;
-    r = horner(c, L);
-  } else {
-    constexpr float c[COPES_NORMAL_TAIL_DEGREE + 1] = COPES_NORMAL_TAIL_COEFFS;
-    r = horner(c, __fadd_rn(sqrt_approx(-L), -COPES_NORMAL_TAIL_SHIFT));
+// Standard normal from one Philox word w: eps = Phi^-1(u), u = ((w & 0x7FFFFE) | 1) 2^-23.
+// OR-ing those bits (made odd) under the exponent of 2 gives the float 2 + m 2^-22 with m
+// odd, so x = 2u - 1 = that - 3 is exact in one add.  Then
+//   eps = sqrt(2) erfinv(x) = x * R(L),  L = log2(1 - x^2),
+// with R a fitted polynomial in L on the central range and in sqrt(-L) - shift on the tail
+// (coefficients: normal_coeffs.h).  R is evaluated relative to its own value, so eps has
+// a small relative error for every x, including x near 0 (L -> 0) and near +-1.
+//
+// The parts return x and r = scale * R(L) when given coefficients pre-multiplied by
+// scale, so a caller forms scale * eps + b as one fma(r, x, b).
+__device__ __forceinline__ float lattice_x(uint32_t w) {
+  return __fadd_rn(__uint_as_float((w & 0x007FFFFEu) | 0x40000001u), -3.0f);
+}
+
+template <int NT>
+__device__ __forceinline__ float tail_ratio(const float (&tail)[NT], float L) {
+  return horner(tail, __fadd_rn(sqrt_approx(-L), -COPES_NORMAL_TAIL_SHIFT));
+}
+
+// One word.  The tail polynomial runs only when some active lane needs it.
+template <int NC, int NT>
+__device__ __forceinline__ void normal_parts(uint32_t w, const float (&central)[NC],
+                                             const float (&tail)[NT], float &x, float &r) {
+  x = lattice_x(w);
+  const float L = lg2_approx(__fmaf_rn(-x, x, 1.0f));
+  r = horner(central, L);
+  const bool in_tail = L < COPES_NORMAL_L_SPLIT;
+  if (__any_sync(__activemask(), in_tail)) {
+    if (in_tail) r = tail_ratio(tail, L);
   }
+}
+
+// The four words of one Philox block with a single warp vote for the tail (taken by a
+// warp with probability ~6%), so the common path carries no per-normal branch.
+template <int NC, int NT>
+__device__ __forceinline__ void normal_parts4(const uint32_t (&w)[4], const float (&central)[NC],
+                                              const float (&tail)[NT], float (&x)[4],
+                                              float (&r)[4]) {
+  float L[4];
+  bool any_tail = false;
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    x[e] = lattice_x(w[e]);
+    L[e] = lg2_approx(__fmaf_rn(-x[e], x[e], 1.0f));
+    r[e] = horner(central, L[e]);
+    any_tail |= L[e] < COPES_NORMAL_L_SPLIT;
+  }
+  if (__any_sync(__activemask(), any_tail)) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      if (L[e] < COPES_NORMAL_L_SPLIT) r[e] = tail_ratio(tail, L[e]);
+  }
+}
+
+#define COPES_UNIT_COEFFS                                                                     \
+  constexpr float unit_central[COPES_NORMAL_CENTRAL_DEGREE + 1] = COPES_NORMAL_CENTRAL_COEFFS; \
+  constexpr float unit_tail[COPES_NORMAL_TAIL_DEGREE + 1] = COPES_NORMAL_TAIL_COEFFS
+
+__device__ __forceinline__ float normal_from_word(uint32_t w) {
+  COPES_UNIT_COEFFS;
+  float x, r;
+  normal_parts(w, unit_central, unit_tail, x, r);
   return __fmul_rn(x, r);
+}
+
+// eps for the four words of one Philox block.
+__device__ __forceinline__ void normals4(const uint32_t (&w)[4], float (&eps)[4]) {
+  COPES_UNIT_COEFFS;
+  float x[4], r[4];
+  normal_parts4(w, unit_central, unit_tail, x, r);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) eps[e] = __fmul_rn(x[e], r[e]);
 }
 
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {

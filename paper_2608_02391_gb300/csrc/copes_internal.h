@@ -5,6 +5,7 @@
 #include <stdint.h>
 
 #include "../../include/copes.h"
+#include "normal_coeffs.h"
 
 namespace copes {
 
@@ -41,6 +42,38 @@ __host__ __device__ __forceinline__ void philox4x32_10(uint32_t c0, uint32_t c1,
   out[3] = c3;
 }
 
+// Round keys of Philox4x32-10: rk[2r] = k0 + r W0, rk[2r+1] = k1 + r W1 (r = 0..9).
+__host__ __device__ __forceinline__ void philox_round_keys(uint32_t k0, uint32_t k1, uint32_t rk[20]) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    rk[2 * r] = k0 + (uint32_t)r * kPhiloxW0;
+    rk[2 * r + 1] = k1 + (uint32_t)r * kPhiloxW1;
+  }
+}
+
+// The same generator with the key schedule precomputed: the per-round key additions
+// are taken out of the hot loop (rk may live in the constant bank or shared memory).
+template <typename RK>
+__host__ __device__ __forceinline__ void philox4x32_10_rk(uint32_t c0, uint32_t c1, uint32_t c2,
+                                                          uint32_t c3, const RK &rk,
+                                                          uint32_t out[4]) {
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    const uint64_t p0 = (uint64_t)kPhiloxM0 * c0;
+    const uint64_t p1 = (uint64_t)kPhiloxM1 * c2;
+    const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ rk[2 * r];
+    const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ rk[2 * r + 1];
+    c1 = (uint32_t)p1;
+    c3 = (uint32_t)p0;
+    c0 = n0;
+    c2 = n2;
+  }
+  out[0] = c0;
+  out[1] = c1;
+  out[2] = c2;
+  out[3] = c3;
+}
+
 // Device error bits (set with atomicOr by a kernel that skipped an access).
 enum : unsigned {
   kErrTileRange = 1u,   // a tile outside [0, n_alloc) or longer than COPES_TILE_MAX
@@ -49,6 +82,12 @@ enum : unsigned {
 };
 
 // ---------------------------------------------------------------- launch arguments
+// R's coefficients pre-multiplied by the perturbation scale (filled by the host).
+struct ScaledCoeffs {
+  float central[COPES_NORMAL_CENTRAL_DEGREE + 1];
+  float tail[COPES_NORMAL_TAIL_DEGREE + 1];
+};
+
 struct ElemArgs {
   void *w;
   float *master;
@@ -61,6 +100,8 @@ struct ElemArgs {
   uint32_t tag;
   float a;  // perturb: signed sigma; init: scale
   float b;  // init: mean
+  ScaledCoeffs coeffs;  // a * R's coefficients (perturb, init)
+  uint32_t rk[20];      // Philox round keys of (seed_lo, seed_hi)
 };
 
 enum ElemOp { kOpPerturb = 0, kOpRestore = 1, kOpInit = 2 };

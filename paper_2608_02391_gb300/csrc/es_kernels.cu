@@ -42,13 +42,19 @@ struct WStore<float> {
   }
 };
 
+// scale * eps + b for one word, with scale folded into the coefficients: one fma.
+__device__ __forceinline__ float scaled_normal_plus(uint32_t w, const ScaledCoeffs &k, float b) {
+  float x, r;
+  normal_parts(w, k.central, k.tail, x, r);
+  return __fmaf_rn(r, x, b);
+}
+
 // Noise for the group at 4q under (k0, k1, tag): four normals.
 __device__ __forceinline__ void group_noise(uint64_t q, uint32_t tag, uint32_t k0, uint32_t k1,
-                                            float eps[4]) {
+                                            float (&eps)[4]) {
   uint32_t x[4];
   philox4x32_10((uint32_t)q, (uint32_t)(q >> 32), 0u, tag, k0, k1, x);
-#pragma unroll
-  for (int e = 0; e < 4; ++e) eps[e] = normal_from_word(x[e]);
+  normals4(x, eps);
 }
 
 // Noise for a single index g: the one word of its counter that g uses.
@@ -63,28 +69,60 @@ __device__ __forceinline__ float index_noise(uint64_t g, uint32_t tag, uint32_t 
 
 // ------------------------------------------------------------ perturb / restore / init
 template <int OP>
+constexpr uint32_t op_tag() { return OP == kOpInit ? COPES_TAG_INIT : COPES_TAG_NOISE; }
+
+// perturb: v = theta + a eps;  init: v = b + a eps;  restore: v = theta.
+template <int OP>
 __device__ __forceinline__ void elem_values(const ElemArgs &a, uint64_t g4, const float th[4],
                                             float v[4]) {
   if (OP == kOpRestore) {
 #pragma unroll
     for (int e = 0; e < 4; ++e) v[e] = th[e];
   } else {
-    float eps[4];
-    group_noise(g4 >> 2, a.tag, a.seed_lo, a.seed_hi, eps);
+    uint32_t w[4];
+    const uint64_t q = g4 >> 2;
+    philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, op_tag<OP>(), a.rk, w);
+    float x[4], r[4];
+    normal_parts4(w, a.coeffs.central, a.coeffs.tail, x, r);  // r = a * R(L)
 #pragma unroll
-    for (int e = 0; e < 4; ++e)
-      v[e] = (OP == kOpPerturb) ? __fmaf_rn(a.a, eps[e], th[e]) : __fmaf_rn(a.a, eps[e], a.b);
+    for (int e = 0; e < 4; ++e) v[e] = __fmaf_rn(r[e], x[e], OP == kOpPerturb ? th[e] : a.b);
   }
 }
 
+// Tile whose ends are multiples of 4: every group is whole.  Tile-local pointers and
+// 32-bit offsets; G groups per thread per step, loads issued before the math.
 template <int OP, typename WT, int G>
-__global__ void __launch_bounds__(kThreads) elem_tiles_kernel(const ElemArgs a) {
-  const uint64_t t = blockIdx.x;
-  const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
-  if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
-    if (threadIdx.x == 0) flag_error(kErrTileRange);
-    return;
+__device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b, uint32_t len) {
+  float *__restrict__ mt = a.master + b;
+  const uint64_t q0 = b >> 2;
+  for (uint32_t off = 4u * threadIdx.x; off < len; off += 4u * kThreads * G) {
+    float th[G][4];
+#pragma unroll
+    for (int i = 0; i < G; ++i) {
+      const uint32_t o = off + 4u * kThreads * i;
+      if (OP != kOpInit && o < len) {
+        const float4 v = ld_stream_f4(mt + o);
+        th[i][0] = v.x, th[i][1] = v.y, th[i][2] = v.z, th[i][3] = v.w;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) th[i][k] = 0.0f;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < G; ++i) {
+      const uint32_t o = off + 4u * kThreads * i;
+      if (o >= len) continue;
+      float v[4];
+      elem_values<OP>(a, (q0 + (o >> 2)) << 2, th[i], v);
+      if (OP == kOpInit) st_stream_f4(mt + o, make_float4(v[0], v[1], v[2], v[3]));
+      WStore<WT>::full(a.w, b + o, v);
+    }
   }
+}
+
+// General tile: groups cut by the tile's ends are handled element by element.
+template <int OP, typename WT, int G>
+__device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, uint64_t e) {
   float *__restrict__ master = a.master;
   const uint64_t lo = b & ~3ull;
   for (uint64_t base = lo + 4ull * threadIdx.x; base < e; base += 4ull * kThreads * G) {
@@ -131,6 +169,19 @@ __global__ void __launch_bounds__(kThreads) elem_tiles_kernel(const ElemArgs a) 
   }
 }
 
+// One block per tile [tiles[2t], tiles[2t+1]).
+template <int OP, typename WT, int G>
+__global__ void __launch_bounds__(kThreads) elem_tiles_kernel(const ElemArgs a) {
+  const uint64_t t = blockIdx.x;
+  const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
+  if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
+    if (threadIdx.x == 0) flag_error(kErrTileRange);
+    return;
+  }
+  if (((b | e) & 3ull) == 0) elem_tile_aligned<OP, WT, G>(a, b, (uint32_t)(e - b));
+  else elem_tile_ragged<OP, WT, G>(a, b, e);
+}
+
 template <int OP, typename WT>
 __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) {
   constexpr int U = 4;
@@ -159,8 +210,12 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
       if (OP == kOpRestore) {
         v = th[u];
       } else {
-        const float eps = index_noise((uint64_t)g[u], a.tag, a.seed_lo, a.seed_hi);
-        v = (OP == kOpPerturb) ? __fmaf_rn(a.a, eps, th[u]) : __fmaf_rn(a.a, eps, a.b);
+        uint32_t x[4];
+        const uint64_t q = (uint64_t)g[u] >> 2;
+        philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, op_tag<OP>(), a.rk, x);
+        const uint32_t s = (uint32_t)g[u] & 3u;
+        const uint32_t wd = s == 0 ? x[0] : (s == 1 ? x[1] : (s == 2 ? x[2] : x[3]));
+        v = scaled_normal_plus(wd, a.coeffs, OP == kOpPerturb ? th[u] : a.b);
       }
       if (OP == kOpInit) master[g[u]] = v;
       WStore<WT>::one(a.w, (uint64_t)g[u], v);
@@ -172,7 +227,7 @@ template <int OP, typename WT>
 static cudaError_t launch_elem_typed(int kind, const ElemArgs &a, cudaStream_t s) {
   if (kind == COPES_SUBSPACE_TILES) {
     if (a.n_tiles == 0) return cudaSuccess;
-    constexpr int G = (OP == kOpRestore) ? 4 : 2;
+    constexpr int G = 4;
     elem_tiles_kernel<OP, WT, G><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
   } else {
     if (a.n_index == 0) return cudaSuccess;
@@ -201,8 +256,10 @@ cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, c
 //   w_j = sum_{i : noise(i) = j} sign_i f_i  (member order, fp32),
 // then every thread regenerates all P noise vectors for its groups in registers and
 // accumulates acc = sum_j w_j eps_j (j ascending), theta = fma(coef, acc, theta).
-__device__ __forceinline__ void noise_weights_to_smem(const UpdateArgs &a, float *s_w) {
+__device__ __forceinline__ void noise_weights_to_smem(const UpdateArgs &a, float *s_w,
+                                                      uint32_t (*s_rk)[20]) {
   for (int j = threadIdx.x; j < a.n_noise; j += blockDim.x) {
+    philox_round_keys(a.seed_lo[j], a.seed_hi[j], s_rk[j]);
     float acc = 0.0f;
     for (int m = a.noise_ptr[j]; m < a.noise_ptr[j + 1]; ++m) {
       const int i = a.noise_member[m];
@@ -217,7 +274,8 @@ __device__ __forceinline__ void noise_weights_to_smem(const UpdateArgs &a, float
 template <typename WT, int G, bool COMMIT>
 __global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
   __shared__ float s_w[COPES_MAX_NOISE];
-  noise_weights_to_smem(a, s_w);
+  __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
+  noise_weights_to_smem(a, s_w, s_rk);
   const uint64_t t = blockIdx.x;
   const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
   if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
@@ -246,12 +304,20 @@ __global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_con
       for (int k = 0; k < 4; ++k) acc[i][k] = 0.0f;
     }
     for (int j = 0; j < P; ++j) {
-      const uint32_t k0 = a.seed_lo[j], k1 = a.seed_hi[j];
+      uint32_t rk[20];
+#pragma unroll
+      for (int r = 0; r < 20; r += 4) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(&s_rk[j][r]);
+        rk[r] = v.x, rk[r + 1] = v.y, rk[r + 2] = v.z, rk[r + 3] = v.w;
+      }
       const float wj = s_w[j];
 #pragma unroll
       for (int i = 0; i < G; ++i) {
         float eps[4];
-        group_noise((base + 4ull * kThreads * i) >> 2, COPES_TAG_NOISE, k0, k1, eps);
+        const uint64_t q = (base + 4ull * kThreads * i) >> 2;
+        uint32_t w[4];
+        philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, w);
+        normals4(w, eps);
 #pragma unroll
         for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
       }
@@ -281,9 +347,10 @@ __global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_con
 }
 
 template <typename WT, bool COMMIT>
-__global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_constant__ UpdateArgs a) {
+__global__ void __launch_bounds__(kThreads, 4) update_index_kernel(const __grid_constant__ UpdateArgs a) {
   __shared__ float s_w[COPES_MAX_NOISE];
-  noise_weights_to_smem(a, s_w);
+  __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
+  noise_weights_to_smem(a, s_w, s_rk);
   constexpr int U = 2;
   const uint64_t s0 = (uint64_t)blockIdx.x * kIndexSegment;
   const uint64_t s1 = min(s0 + (uint64_t)kIndexSegment, a.n_index);
@@ -306,11 +373,22 @@ __global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_con
       acc[u] = 0.0f;
     }
     for (int j = 0; j < P; ++j) {
-      const uint32_t k0 = a.seed_lo[j], k1 = a.seed_hi[j];
+      uint32_t rk[20];
+#pragma unroll
+      for (int r = 0; r < 20; r += 4) {
+        const uint4 v = *reinterpret_cast<const uint4 *>(&s_rk[j][r]);
+        rk[r] = v.x, rk[r + 1] = v.y, rk[r + 2] = v.z, rk[r + 3] = v.w;
+      }
       const float wj = s_w[j];
 #pragma unroll
-      for (int u = 0; u < U; ++u)
-        acc[u] = __fmaf_rn(wj, index_noise((uint64_t)g[u], COPES_TAG_NOISE, k0, k1), acc[u]);
+      for (int u = 0; u < U; ++u) {
+        uint32_t x[4];
+        const uint64_t q = (uint64_t)g[u] >> 2;
+        philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, x);
+        const uint32_t s = (uint32_t)g[u] & 3u;
+        const uint32_t wd = s == 0 ? x[0] : (s == 1 ? x[1] : (s == 2 ? x[2] : x[3]));
+        acc[u] = __fmaf_rn(wj, normal_from_word(wd), acc[u]);
+      }
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
@@ -326,7 +404,7 @@ template <typename WT, bool COMMIT>
 static cudaError_t launch_update_typed(int kind, const UpdateArgs &a, cudaStream_t s) {
   if (kind == COPES_SUBSPACE_TILES) {
     if (a.n_tiles == 0) return cudaSuccess;
-    update_tiles_kernel<WT, 2, COMMIT><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+    update_tiles_kernel<WT, 4, COMMIT><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
   } else {
     if (a.n_index == 0) return cudaSuccess;
     const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
@@ -349,9 +427,9 @@ __global__ void debug_philox_kernel(uint64_t seed, uint64_t q0, uint64_t n, uint
   const uint64_t i = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const uint64_t q = q0 + i;
-  uint32_t x[4];
-  philox4x32_10((uint32_t)q, (uint32_t)(q >> 32), aux, tag, (uint32_t)seed,
-                (uint32_t)(seed >> 32), x);
+  uint32_t rk[20], x[4];
+  philox_round_keys((uint32_t)seed, (uint32_t)(seed >> 32), rk);
+  philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), aux, tag, rk, x);
   reinterpret_cast<uint4 *>(out)[i] = make_uint4(x[0], x[1], x[2], x[3]);
 }
 

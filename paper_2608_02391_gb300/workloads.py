@@ -187,6 +187,12 @@ def workload(name: str) -> Workload:
         ts = qwen_8b_tensors()
         return Workload("8b", ts, K=4, mode="groups", n_members=128, sigma=5e-4, alpha=5e-4,
                         shaping="zscore", group_of=group_by_type(ts), cycles=10, data_seed=37)
+    if name == "4b-slice":
+        # profiling case: the 4B workload's step on 4 tensors of 2^26 parameters (1.6 GB
+        # resident: larger than L2, small enough for multi-pass counter captures)
+        ts = [Tensor(f"block{i}", 1 << 26, "attn", i) for i in range(4)]
+        return Workload("4b-slice", ts, K=4, mode="groups", n_members=32, sigma=1e-3, alpha=5e-4,
+                        shaping="zscore", group_of=[0, 1, 2, 3], data_seed=35)
     raise KeyError(name)
 
 

@@ -38,11 +38,14 @@ def test_philox_known_answer_vectors(copes):
 
 
 def test_transform_exhaustive(copes):
-    """Every distinct uniform the transform can see: words m << 9, m < 2^23."""
-    m = torch.arange(1 << 23, dtype=torch.int64, device="cuda")
-    words = (m << 9).to(torch.int32)  # two's-complement wrap keeps the bit pattern
+    """Every distinct uniform the transform can see: words 2m, m < 2^22 (bits 1..22),
+    plus the same words with the ignored bits set."""
+    m = torch.arange(1 << 22, dtype=torch.int64, device="cuda")
+    words = (2 * m).to(torch.int32)
     got = copes.debug_transform(words).cpu().numpy().astype(np.float64)
-    u = (2.0 * np.arange(1 << 23, dtype=np.float64) + 1.0) * 2.0**-24
+    noisy = (2 * m + 1 + (0x1FF << 23)).to(torch.int32)  # bit 0 and bits 23..31 set
+    assert np.array_equal(copes.debug_transform(noisy).cpu().numpy().astype(np.float64), got)
+    u = (2.0 * np.arange(1 << 22, dtype=np.float64) + 1.0) * 2.0**-23
     ref = oracle.normal_quantile_array(u)
     assert_normals_close(got, ref)
     rel = np.abs(got - ref) / np.abs(ref)

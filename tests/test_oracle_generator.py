@@ -93,23 +93,25 @@ def test_philox_matches_curand_host_generator():
 
 def test_uniform_exact_odd_multiples():
     rng = np.random.default_rng(1)
-    xs = [0, 1, 255, 256, 0x7FFFFFFF, 0x80000000, 0xFFFFFFFF] + [
+    xs = [0, 1, 2, 255, 256, 0x7FFFFE, 0x7FFFFF, 0x800000, 0xFFFFFFFF] + [
         int(x) for x in rng.integers(0, 2**32, size=2000, dtype=np.uint64)]
     for x in xs:
         u = oracle.uniform(x)
-        frac = Fraction(u) * (1 << 24)
+        frac = Fraction(u) * (1 << 23)
         assert frac.denominator == 1 and frac.numerator % 2 == 1
-        assert frac.numerator == ((x >> 8) | 1)
+        assert frac.numerator == ((x % (1 << 23)) | 1)  # bits 1..22 of the word, made odd
         assert 0.0 < u < 1.0
         assert np.float32(u) == u  # exact in fp32
-    assert oracle.uniform(0) == 2.0**-24
-    assert oracle.uniform(0xFFFFFFFF) == 1.0 - 2.0**-24
+    assert oracle.uniform(0) == 2.0**-23
+    assert oracle.uniform(0xFFFFFFFF) == 1.0 - 2.0**-23
+    # only bits 1..22 matter
+    assert oracle.uniform(0xFF800000 | 0x1234) == oracle.uniform(0x1235)
 
 
 def test_quantile_exhaustive_against_scipy():
-    """All 2^23 values the transform can see, against scipy.special.ndtri."""
-    m = np.arange(1 << 23, dtype=np.float64)
-    u = (2.0 * m + 1.0) * 2.0**-24
+    """All 2^22 values the transform can see, against scipy.special.ndtri."""
+    m = np.arange(1 << 22, dtype=np.float64)
+    u = (2.0 * m + 1.0) * 2.0**-23
     oracle.clear_fault()
     q = oracle.normal_quantile_array(u)
     assert oracle.fault_flag() == 0
@@ -131,7 +133,7 @@ def test_noise_composition_matches_independent_pieces():
     eps = oracle.noise(seed, g)
     for gi, e in zip(g.tolist(), eps.tolist()):
         w = philox_bigint.words(seed, gi >> 2)[gi & 3]
-        u = ((w >> 8) | 1) * 2.0**-24
+        u = ((w & 0x7FFFFE) | 1) * 2.0**-23
         assert abs(e - special.ndtri(u)) <= 1e-13 * max(1.0, abs(e))
 
 
