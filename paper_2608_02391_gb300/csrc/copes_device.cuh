@@ -69,15 +69,14 @@ __device__ __forceinline__ void normal_parts4(const uint32_t (&w)[4], const floa
                                               const float (&tail)[NT], float (&x)[4],
                                               float (&r)[4]) {
   float L[4];
-  bool any_tail = false;
 #pragma unroll
   for (int e = 0; e < 4; ++e) {
     x[e] = lattice_x(w[e]);
     L[e] = lg2_approx(__fmaf_rn(-x[e], x[e], 1.0f));
     r[e] = horner(central, L[e]);
-    any_tail |= L[e] < COPES_NORMAL_L_SPLIT;
   }
-  if (__any_sync(__activemask(), any_tail)) {
+  const float L_min = fminf(fminf(L[0], L[1]), fminf(L[2], L[3]));
+  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
 #pragma unroll
     for (int e = 0; e < 4; ++e)
       if (L[e] < COPES_NORMAL_L_SPLIT) r[e] = tail_ratio(tail, L[e]);

@@ -71,17 +71,17 @@ __device__ __forceinline__ float index_noise(uint64_t g, uint32_t tag, uint32_t 
 template <int OP>
 constexpr uint32_t op_tag() { return OP == kOpInit ? COPES_TAG_INIT : COPES_TAG_NOISE; }
 
-// perturb: v = theta + a eps;  init: v = b + a eps;  restore: v = theta.
+// perturb: v = theta + a eps;  init: v = b + a eps;  restore: v = theta.  (q_lo, q_hi) is
+// the group's Philox counter g4 >> 2.
 template <int OP>
-__device__ __forceinline__ void elem_values(const ElemArgs &a, uint64_t g4, const float th[4],
-                                            float v[4]) {
+__device__ __forceinline__ void elem_values(const ElemArgs &a, uint32_t q_lo, uint32_t q_hi,
+                                            const float th[4], float v[4]) {
   if (OP == kOpRestore) {
 #pragma unroll
     for (int e = 0; e < 4; ++e) v[e] = th[e];
   } else {
     uint32_t w[4];
-    const uint64_t q = g4 >> 2;
-    philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, op_tag<OP>(), a.rk, w);
+    philox4x32_10_rk(q_lo, q_hi, 0u, op_tag<OP>(), a.rk, w);
     float x[4], r[4];
     normal_parts4(w, a.coeffs.central, a.coeffs.tail, x, r);  // r = a * R(L)
 #pragma unroll
@@ -91,10 +91,14 @@ __device__ __forceinline__ void elem_values(const ElemArgs &a, uint64_t g4, cons
 
 // Tile whose ends are multiples of 4: every group is whole.  Tile-local pointers and
 // 32-bit offsets; G groups per thread per step, loads issued before the math.
-template <int OP, typename WT, int G>
+// HI0: every counter of the tile is below 2^32 (its high word is the constant 0), so the
+// counter arithmetic stays in 32 bits and the compiler drops Philox's first-round
+// multiply of word 2 and hoists the second round's multiply of word 0.
+template <int OP, typename WT, int G, bool HI0>
 __device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b, uint32_t len) {
   float *__restrict__ mt = a.master + b;
   const uint64_t q0 = b >> 2;
+  const uint32_t q0_lo = (uint32_t)q0;
   for (uint32_t off = 4u * threadIdx.x; off < len; off += 4u * kThreads * G) {
     float th[G][4];
 #pragma unroll
@@ -113,7 +117,12 @@ __device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b,
       const uint32_t o = off + 4u * kThreads * i;
       if (o >= len) continue;
       float v[4];
-      elem_values<OP>(a, (q0 + (o >> 2)) << 2, th[i], v);
+      if (HI0) {
+        elem_values<OP>(a, q0_lo + (o >> 2), 0u, th[i], v);
+      } else {
+        const uint64_t q = q0 + (o >> 2);
+        elem_values<OP>(a, (uint32_t)q, (uint32_t)(q >> 32), th[i], v);
+      }
       if (OP == kOpInit) st_stream_f4(mt + o, make_float4(v[0], v[1], v[2], v[3]));
       WStore<WT>::full(a.w, b + o, v);
     }
@@ -151,7 +160,7 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
       const uint64_t g4 = base + 4ull * kThreads * i;
       if (g4 >= e) continue;
       float v[4];
-      elem_values<OP>(a, g4, th[i], v);
+      elem_values<OP>(a, (uint32_t)(g4 >> 2), (uint32_t)(g4 >> 34), th[i], v);
       if (full[i]) {
         if (OP == kOpInit) st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
         WStore<WT>::full(a.w, g4, v);
@@ -178,8 +187,12 @@ __global__ void __launch_bounds__(kThreads) elem_tiles_kernel(const ElemArgs a) 
     if (threadIdx.x == 0) flag_error(kErrTileRange);
     return;
   }
-  if (((b | e) & 3ull) == 0) elem_tile_aligned<OP, WT, G>(a, b, (uint32_t)(e - b));
-  else elem_tile_ragged<OP, WT, G>(a, b, e);
+  if (((b | e) & 3ull) == 0) {
+    if ((e >> 34) == 0) elem_tile_aligned<OP, WT, G, true>(a, b, (uint32_t)(e - b));
+    else elem_tile_aligned<OP, WT, G, false>(a, b, (uint32_t)(e - b));
+  } else {
+    elem_tile_ragged<OP, WT, G>(a, b, e);
+  }
 }
 
 template <int OP, typename WT>
@@ -271,6 +284,10 @@ __device__ __forceinline__ void noise_weights_to_smem(const UpdateArgs &a, float
   __syncthreads();
 }
 
+template <typename WT, int G, bool COMMIT, bool HI0>
+__device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_w,
+                                            const uint32_t (*s_rk)[20], uint64_t b, uint64_t e);
+
 template <typename WT, int G, bool COMMIT>
 __global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
   __shared__ float s_w[COPES_MAX_NOISE];
@@ -282,6 +299,15 @@ __global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_con
     if (threadIdx.x == 0) flag_error(kErrTileRange);
     return;
   }
+  if ((e >> 34) == 0) update_tile<WT, G, COMMIT, true>(a, s_w, s_rk, b, e);
+  else update_tile<WT, G, COMMIT, false>(a, s_w, s_rk, b, e);
+}
+
+// Members folded into noise weights s_w and round keys s_rk per noise vector; this
+// block's tile [b, e).  HI0 as in elem_values.
+template <typename WT, int G, bool COMMIT, bool HI0>
+__device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_w,
+                                            const uint32_t (*s_rk)[20], uint64_t b, uint64_t e) {
   float *__restrict__ master = a.master;
   const uint64_t lo = b & ~3ull;
   const int P = a.n_noise;
@@ -303,6 +329,7 @@ __global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_con
 #pragma unroll
       for (int k = 0; k < 4; ++k) acc[i][k] = 0.0f;
     }
+    const uint32_t q_lo = (uint32_t)(base >> 2);  // counter of group 0 (HI0: the whole counter)
     for (int j = 0; j < P; ++j) {
       uint32_t rk[20];
 #pragma unroll
@@ -314,9 +341,13 @@ __global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_con
 #pragma unroll
       for (int i = 0; i < G; ++i) {
         float eps[4];
-        const uint64_t q = (base + 4ull * kThreads * i) >> 2;
         uint32_t w[4];
-        philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, w);
+        if (HI0) {
+          philox4x32_10_rk(q_lo + kThreads * i, 0u, 0u, COPES_TAG_NOISE, rk, w);
+        } else {
+          const uint64_t q = (base >> 2) + kThreads * i;
+          philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, w);
+        }
         normals4(w, eps);
 #pragma unroll
         for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
