@@ -109,6 +109,19 @@ ElemArgs elem_args(const copes_params *p, const copes_subspace *S) {
   return a;
 }
 
+// R's coefficients times scale, plus the packed (c, c) pairs of the central polynomial.
+void scaled_coeffs(float scale, copes::ScaledCoeffs &k) {
+  static const float central[] = COPES_NORMAL_CENTRAL_COEFFS;
+  static const float tail[] = COPES_NORMAL_TAIL_COEFFS;
+  for (int i = 0; i <= COPES_NORMAL_CENTRAL_DEGREE; ++i) {
+    k.central[i] = scale * central[i];
+    uint32_t bits;
+    memcpy(&bits, &k.central[i], 4);
+    k.central2[i] = (unsigned long long)bits | ((unsigned long long)bits << 32);
+  }
+  for (int i = 0; i <= COPES_NORMAL_TAIL_DEGREE; ++i) k.tail[i] = scale * tail[i];
+}
+
 int run_elementwise(int op, const copes_params *p, const copes_subspace *S, uint64_t seed,
                     uint32_t tag, float a_val, float b_val, cudaStream_t s, const char *who) {
   int rc = check_params(p, who);
@@ -121,10 +134,7 @@ int run_elementwise(int op, const copes_params *p, const copes_subspace *S, uint
   a.a = a_val;
   a.b = b_val;
   // the scale folded into the normal's polynomial: a * eps = x * (a * R(L))
-  static const float central[] = COPES_NORMAL_CENTRAL_COEFFS;
-  static const float tail[] = COPES_NORMAL_TAIL_COEFFS;
-  for (int i = 0; i <= COPES_NORMAL_CENTRAL_DEGREE; ++i) a.coeffs.central[i] = a_val * central[i];
-  for (int i = 0; i <= COPES_NORMAL_TAIL_DEGREE; ++i) a.coeffs.tail[i] = a_val * tail[i];
+  scaled_coeffs(a_val, a.coeffs);
   copes::philox_round_keys(a.seed_lo, a.seed_hi, a.rk);
   return launch_status(copes::launch_elementwise(op, S->kind, p->dtype, a, s), who);
 }

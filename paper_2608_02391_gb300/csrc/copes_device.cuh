@@ -83,6 +83,52 @@ __device__ __forceinline__ void normal_parts4(const uint32_t (&w)[4], const floa
   }
 }
 
+// Packed fp32 pairs: one fma.rn.f32x2 performs the two lanes' fp32 fmas, each rounded
+// exactly as a scalar fma, at half the instruction count.
+__device__ __forceinline__ unsigned long long pack_f32x2(float lo, float hi) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpack_f32x2(unsigned long long v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ unsigned long long fma_f32x2(unsigned long long a, unsigned long long b,
+                                                        unsigned long long c) {
+  unsigned long long d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+
+// normal_parts4 with the central polynomial evaluated on two pairs of normals; central2
+// holds each coefficient twice (c, c).  Same results as normal_parts4, bit for bit.
+template <int NC, int NT>
+__device__ __forceinline__ void normal_parts4_x2(const uint32_t (&w)[4],
+                                                 const unsigned long long (&central2)[NC],
+                                                 const float (&tail)[NT], float (&x)[4],
+                                                 float (&r)[4]) {
+  float L[4];
+#pragma unroll
+  for (int e = 0; e < 4; ++e) {
+    x[e] = lattice_x(w[e]);
+    L[e] = lg2_approx(__fmaf_rn(-x[e], x[e], 1.0f));
+  }
+#pragma unroll
+  for (int p = 0; p < 2; ++p) {
+    const unsigned long long Lp = pack_f32x2(L[2 * p], L[2 * p + 1]);
+    unsigned long long acc = central2[NC - 1];
+#pragma unroll
+    for (int i = NC - 2; i >= 0; --i) acc = fma_f32x2(acc, Lp, central2[i]);
+    unpack_f32x2(acc, r[2 * p], r[2 * p + 1]);
+  }
+  const float L_min = fminf(fminf(L[0], L[1]), fminf(L[2], L[3]));
+  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e)
+      if (L[e] < COPES_NORMAL_L_SPLIT) r[e] = tail_ratio(tail, L[e]);
+  }
+}
+
 #define COPES_UNIT_COEFFS                                                                     \
   constexpr float unit_central[COPES_NORMAL_CENTRAL_DEGREE + 1] = COPES_NORMAL_CENTRAL_COEFFS; \
   constexpr float unit_tail[COPES_NORMAL_TAIL_DEGREE + 1] = COPES_NORMAL_TAIL_COEFFS

@@ -84,6 +84,7 @@ enum : unsigned {
 // ---------------------------------------------------------------- launch arguments
 // R's coefficients pre-multiplied by the perturbation scale (filled by the host).
 struct ScaledCoeffs {
+  unsigned long long central2[COPES_NORMAL_CENTRAL_DEGREE + 1];  // (c, c) pairs
   float central[COPES_NORMAL_CENTRAL_DEGREE + 1];
   float tail[COPES_NORMAL_TAIL_DEGREE + 1];
 };

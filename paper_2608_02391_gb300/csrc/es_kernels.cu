@@ -83,7 +83,7 @@ __device__ __forceinline__ void elem_values(const ElemArgs &a, uint32_t q_lo, ui
     uint32_t w[4];
     philox4x32_10_rk(q_lo, q_hi, 0u, op_tag<OP>(), a.rk, w);
     float x[4], r[4];
-    normal_parts4(w, a.coeffs.central, a.coeffs.tail, x, r);  // r = a * R(L)
+    normal_parts4_x2(w, a.coeffs.central2, a.coeffs.tail, x, r);  // r = a * R(L)
 #pragma unroll
     for (int e = 0; e < 4; ++e) v[e] = __fmaf_rn(r[e], x[e], OP == kOpPerturb ? th[e] : a.b);
   }
@@ -348,6 +348,8 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
           const uint64_t q = (base >> 2) + kThreads * i;
           philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, w);
         }
+        // scalar Horner here: the packed form needs the coefficient pairs in registers,
+        // which costs this kernel more occupancy than it saves in issue slots
         normals4(w, eps);
 #pragma unroll
         for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
