@@ -1,0 +1,306 @@
+"""Parity at the workloads' full sizes, in the launch configuration the benchmark times.
+
+The oracle computes sampled outputs element by element. Samples include every subspace
+range's first and last elements and random interior ones. Inputs come from seeded
+generators: numpy for the tiny vector, torch's seeded CUDA generator for the large
+arenas. The rewards are seeded synthetic scalars shared by both sides. Size-independent
+properties are checked on the whole subspace: restore is exact, and elements outside S
+are untouched.
+"""
+import gc
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_02391_gb300 import workloads as wl
+from tolerances import (assert_bf16_close, assert_fitness_close, assert_perturb_fp32_close,
+                        assert_update_close)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def copes():
+    from paper_2608_02391_gb300 import copes as c
+    c.load()
+    return c
+
+
+@pytest.fixture(autouse=True)
+def free_memory():
+    yield
+    gc.collect()
+    torch.cuda.empty_cache()
+
+
+SHAPE = {"zscore": oracle.SHAPE_ZSCORE, "centered_rank": oracle.SHAPE_CENTERED_RANK,
+         "zscore_grouped": oracle.SHAPE_ZSCORE_GROUPED, "none": oracle.SHAPE_NONE}
+
+
+def make_arena(copes, w: wl.Workload, seed=0):
+    """fp32 master ~ N(0, 0.02^2) from torch's seeded CUDA generator, norms = 1.0, and
+    w = bf16(master)."""
+    layout = copes.Layout(w.numel)
+    master = torch.empty(layout.d_pad, dtype=torch.float32, device="cuda")
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(seed)
+    master.normal_(0.0, w.init_scale, generator=gen)
+    off = layout.offsets
+    for t, ten in enumerate(w.tensors):
+        if ten.kind == "norm":
+            master[int(off[t]):int(off[t]) + ten.numel].fill_(1.0)
+    return copes.Arena(master.to(torch.bfloat16), master), layout
+
+
+def sample_from_ranges(ranges, n_random, rng):
+    edges = []
+    for b, e in ranges:
+        edges += [b, min(b + 1, e - 1), max(e - 2, b), e - 1]
+    sizes = np.array([e - b for b, e in ranges], dtype=np.float64)
+    pick = rng.choice(len(ranges), size=n_random, p=sizes / sizes.sum())
+    rnd = [int(ranges[i][0] + rng.integers(0, ranges[i][1] - ranges[i][0])) for i in pick]
+    return np.unique(np.array(edges + rnd, dtype=np.int64))
+
+
+def tile_ranges(sub):
+    t = sub.tensor.cpu().numpy()
+    out = []
+    for b, e in t:
+        if out and out[-1][1] == int(b):
+            out[-1] = (out[-1][0], int(e))
+        else:
+            out.append((int(b), int(e)))
+    return out
+
+
+def bf16_bits_of(t: torch.Tensor, idx: np.ndarray):
+    return t.view(torch.int16)[torch.from_numpy(idx).cuda()].cpu().numpy().view(np.uint16)
+
+
+def check_visit(copes, arena, sub, sample, w: wl.Workload, k, iteration, rewards, pairing=None,
+                check_members=(0, 1)):
+    """One round-robin visit on the GPU; the oracle recomputes the sampled outputs."""
+    pairing = copes.ANTITHETIC if pairing is None else pairing
+    N = w.n_members
+    nid, sign, P = copes.member_table(N, pairing)
+    seeds = copes.member_seeds(w.base_seed, iteration, k, P)
+    sigma = np.float32(w.sigma)
+    idx_t = torch.from_numpy(sample).cuda()
+    theta = arena.master[idx_t].cpu().numpy()
+    g = sample.astype(np.uint64)
+    w_outside_sum = None
+    for i in range(N):
+        copes.perturb(arena, sub, int(seeds[nid[i]]), float(sign[i] * sigma))
+        if i in check_members:
+            ref_bits, _ = oracle.perturb_at(g, theta, int(seeds[nid[i]]), float(sign[i] * sigma), oracle.BF16)
+            scale = np.maximum(np.abs(theta), np.abs(sigma * oracle.noise(int(seeds[nid[i]]), g)))
+            assert_bf16_close(bf16_bits_of(arena.w, sample), ref_bits.astype(np.uint16), scale)
+    copes.restore(arena, sub)
+    assert np.array_equal(bf16_bits_of(arena.w, sample), oracle.bf16_bits_array(theta))
+    r_dev = torch.from_numpy(rewards).cuda()
+    f = copes.shape_fitness(r_dev, w.shaping).cpu().numpy()
+    f_ref = oracle.shape_fitness(rewards, SHAPE[w.shaping])
+    assert_fitness_close(f, f_ref)
+    coef = np.float32(copes.step_coef(w.alpha, N, float(sigma), copes.COEF_OPENAI))
+    copes.update(arena, sub, nid, sign, torch.from_numpy(f).cuda(), seeds, float(coef), fuse_commit=True)
+    wj = oracle.noise_weights(nid, sign, f_ref, P)
+    _, exact, scale = oracle.update_at(g, theta, seeds, wj, coef)
+    got = arena.master[idx_t].cpu().numpy()
+    assert_update_close(got, exact, scale)
+    assert np.array_equal(bf16_bits_of(arena.w, sample), oracle.bf16_bits_array(got))
+
+
+def whole_subspace_properties(copes, arena, sub, seed):
+    """Restore after perturb is exact on all of S; elements outside S keep their bits."""
+    before = arena.w.view(torch.int16).clone()
+    copes.perturb(arena, sub, seed, 1e-3)
+    copes.restore(arena, sub)
+    assert torch.equal(arena.w.view(torch.int16), before)
+    del before
+
+
+# ------------------------------------------------------------------------------ tiny
+def test_tiny_round_robin_loop_matches_oracle_trajectory(copes):
+    """The tiny workload end to end: 3 cycles x 4 contiguous subspaces x 8 antithetic
+    members, rewards r_i = c . w_i computed by the oracle from its own perturbed weights.
+    GPU and oracle run independent trajectories from the same rewards. Errors add across a
+    subspace's 3 updates, so the tolerance is the sum of the per-update bounds."""
+    w = wl.workload("tiny")
+    theta0, cvec = wl.tiny_theta_and_objective()
+    n = theta0.size
+    K, N = w.K, w.n_members
+    sigma = np.float32(w.sigma)
+    coef = np.float32(w.alpha / (N * float(sigma)))
+    o_master = theta0.copy()
+    bound = np.zeros(n)
+    g_master = torch.from_numpy(theta0.copy()).cuda()
+    arena = copes.Arena(g_master.clone(), g_master)  # fp32 working tensor
+    layout = copes.Layout([n])
+    nid, sign, P = oracle.member_table(N, oracle.ANTITHETIC)
+    for cycle in range(w.cycles):
+        for k in range(K):
+            ranges = oracle.contiguous_ranges([n], K, k)
+            (b, e), = ranges
+            sub = copes.subspace_build(layout, copes.PART_CONTIGUOUS, K, k, tile_size=1 << 14)
+            assert tile_ranges(sub) == ranges
+            seeds = np.array([oracle.member_seed(w.base_seed, cycle, k, j) for j in range(P)], np.uint64)
+            g = np.arange(b, e, dtype=np.uint64)
+            rewards = np.zeros(N, np.float32)
+            base_dot = float(cvec @ o_master) - float(cvec[b:e] @ o_master[b:e])
+            for i in range(N):
+                _, exact = oracle.perturb_at(g, o_master[b:e], int(seeds[nid[i]]), float(sign[i] * sigma), oracle.FP32)
+                rewards[i] = np.float32(base_dot + float(cvec[b:e] @ exact))
+                copes.perturb(arena, sub, int(seeds[nid[i]]), float(sign[i] * sigma))
+                if i == 0:
+                    got = arena.w[b:e].cpu().numpy()
+                    ref_theta = o_master[b:e]
+                    eps = oracle.noise(int(seeds[nid[i]]), g)
+                    # the GPU perturbs its own master, which differs from the oracle's by the
+                    # bound accumulated so far
+                    tol = 1e-6 * np.maximum.reduce([np.abs(exact), np.abs(ref_theta), np.abs(sigma * eps)]) + bound[b:e]
+                    assert np.all(np.abs(got - exact) <= tol)
+            copes.restore(arena, sub)
+            f_ref = oracle.shape_fitness(rewards, oracle.SHAPE_ZSCORE)
+            f = copes.shape_fitness(torch.from_numpy(rewards).cuda(), "zscore")
+            assert_fitness_close(f.cpu().numpy(), f_ref)
+            copes.update(arena, sub, nid, sign, f, seeds, float(coef), fuse_commit=True)
+            wj = oracle.noise_weights(nid, sign, f_ref, P)
+            _, exact, scale = oracle.update_at(g, o_master[b:e], seeds, wj, coef)
+            o_master[b:e] = exact.astype(np.float32)
+            bound[b:e] += 1e-6 * np.maximum(np.abs(exact), scale)
+            got = g_master[b:e].cpu().numpy()
+            assert np.all(np.abs(got.astype(np.float64) - exact) <= bound[b:e])
+            assert torch.equal(arena.w[b:e], g_master[b:e])  # fp32 commit is a copy
+    copes.check()
+
+
+# ------------------------------------------------------------------------ 0.5B / 4B / 8B
+@pytest.mark.parametrize("name,visits", [("0.5b", range(8)), ("4b", [0, 3, 7])])
+def test_layer_block_workloads_sampled(copes, name, visits):
+    w = wl.workload(name)
+    arena, layout = make_arena(copes, w)
+    rng = np.random.default_rng(5)
+    rewards = wl.reward_stream(w, 8)
+    for k in visits:
+        sub = copes.subspace_build(layout, copes.PART_TENSOR_GROUPS, w.K, k, group_of=w.group_of,
+                                   tile_size=copes.DEFAULT_TILE)
+        ranges = tile_ranges(sub)
+        assert ranges == oracle.group_ranges(w.numel, w.group_of, k)
+        sample = sample_from_ranges(ranges, 4096, rng)
+        check_visit(copes, arena, sub, sample, w, k, 0, rewards[k])
+        if k == visits[0]:
+            whole_subspace_properties(copes, arena, sub, 99)
+    copes.check()
+
+
+def test_8b_type_groups_sampled(copes):
+    w = wl.workload("8b")
+    arena, layout = make_arena(copes, w)
+    rng = np.random.default_rng(8)
+    rewards = wl.reward_stream(w, 4)
+    for k in (0, 2):  # attention (1.51e9 parameters), norms + embeddings
+        sub = copes.subspace_build(layout, copes.PART_TENSOR_GROUPS, w.K, k, group_of=w.group_of,
+                                   tile_size=copes.DEFAULT_TILE)
+        ranges = tile_ranges(sub)
+        assert ranges == oracle.group_ranges(w.numel, w.group_of, k)
+        check_visit(copes, arena, sub, sample_from_ranges(ranges, 4096, rng), w, k, 0, rewards[k],
+                    check_members=(0, 127))
+    copes.check()
+
+
+# ---------------------------------------------------------------------------- 4B hash
+def test_4b_hash_partition_and_gather_visit(copes):
+    w = wl.workload("4b-hash")
+    arena, layout = make_arena(copes, w)
+    tids = list(range(len(w.tensors)))
+    layout = copes.Layout(w.numel, tids)
+    lists = copes.hash_partition(layout, w.K, w.partition_seed)
+    counts = np.array([s.numel for s in lists])
+    assert counts.sum() == w.d
+    sd = np.sqrt(w.d / w.K * (1 - 1 / w.K))
+    assert np.all(np.abs(counts - w.d / w.K) < 5 * sd)
+    for s in lists:
+        assert bool((s.tensor[1:] > s.tensor[:-1]).all())
+    # membership of random elements, from the oracle's hash
+    rng = np.random.default_rng(11)
+    off = oracle.layout(w.numel)
+    for _ in range(2000):
+        t = int(rng.integers(0, len(w.tensors)))
+        e = int(rng.integers(0, w.numel[t]))
+        k = oracle.hash_subspace(w.partition_seed, tids[t], e, w.K)
+        g = int(off[t]) + e
+        pos = int(torch.searchsorted(lists[k].tensor, torch.tensor([g], device="cuda")).item())
+        assert pos < lists[k].numel and int(lists[k].tensor[pos].item()) == g
+    # one gather visit on subspace 3 with the workload's N = 64
+    sub = lists[3]
+    pos = np.unique(np.concatenate([[0, 1, sub.numel - 1], rng.integers(0, sub.numel, 4096)]))
+    sample = sub.tensor[torch.from_numpy(pos).cuda()].cpu().numpy()
+    rewards = wl.reward_stream(w, 4)[3]
+    check_visit(copes, arena, sub, sample, w, 3, 0, rewards)
+    del lists
+    copes.check()
+
+
+# ----------------------------------------------------------- beyond 2^34 global indices
+def test_counters_beyond_2_34(copes):
+    """Tiles past global index 2^34 take the kernels' general counter path; a range
+    crossing the boundary checks both paths against the oracle."""
+    n = (1 << 34) + (1 << 20)
+    master = torch.empty(n, dtype=torch.float32, device="cuda")
+    lo, hi = (1 << 34) - (1 << 19), (1 << 34) + (1 << 19)
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(3)
+    master[lo:hi].normal_(0.0, 0.02, generator=gen)
+    wt = torch.zeros(n, dtype=torch.bfloat16, device="cuda")
+    arena = copes.Arena(wt, master)
+    sub = copes.tiles_from_ranges([(lo, hi)], tile_size=1 << 16)
+    w = wl.Workload("big", [wl.Tensor("x", n, "vector")], K=1, mode="contiguous", n_members=8,
+                    sigma=1e-3, alpha=5e-4, shaping="zscore")
+    rng = np.random.default_rng(4)
+    sample = np.unique(np.concatenate([[lo, (1 << 34) - 1, 1 << 34, hi - 1],
+                                       rng.integers(lo, hi, 4000)])).astype(np.int64)
+    rewards = (rng.integers(0, 17, 8) / 16).astype(np.float32)
+    check_visit(copes, arena, sub, sample, w, 0, 0, rewards)
+    copes.check()
+
+
+# ------------------------------------------------------------------ Algorithm 1 (SYNC)
+@pytest.mark.parametrize("joint", [True, False])
+def test_sync_step_algorithm1_matches_oracle(copes, joint):
+    """Algorithm 1 on a 1M-parameter vector: a random equal-size chunk partition, K = 4,
+    N = 8 (N_k = 2), sigma_k = sqrt(K) sigma (Eq. 11), joint (Eq. 12) or per-subspace
+    standardisation, coefficient alpha / N_k (Eq. 13), every g_k from the same
+    pre-update theta."""
+    from paper_2608_02391_gb300 import es
+    n, K, N, chunk = 1 << 20, 4, 8, 4096
+    theta0, _ = wl.tiny_theta_and_objective()
+    master = torch.from_numpy(theta0.copy()).cuda()
+    arena = copes.Arena(master.to(torch.bfloat16), master)
+    layout = copes.Layout([n])
+    subs = es.build_subspaces(layout, "random_chunks", K, seed=77, chunk=chunk)
+    cmap = oracle.random_chunks(n // chunk, K, 77)
+    for k in range(K):
+        assert tile_ranges(subs[k]) == oracle.chunk_ranges([n], chunk, cmap, k)
+    cfg = es.ESConfig(n_members=N, sigma=1e-3, alpha=5e-4, shaping="zscore",
+                      convention=copes.COEF_PAPER, dimension_aware=True)
+    rewards = (np.random.default_rng(2).integers(0, 17, N) / 16).astype(np.float32)
+    f = es.sync_step(arena, subs, 0, cfg, n, torch.from_numpy(rewards).cuda(), joint=joint)
+    group = np.repeat(np.arange(K), N // K).astype(np.int32)
+    f_ref = (oracle.shape_fitness(rewards, oracle.SHAPE_ZSCORE) if joint
+             else oracle.shape_fitness(rewards, oracle.SHAPE_ZSCORE_GROUPED, group))
+    assert_fitness_close(f.cpu().numpy(), f_ref)
+    nid, sign, P = oracle.member_table(N // K, oracle.ANTITHETIC)
+    got = master.cpu().numpy()
+    for k in range(K):
+        ranges = oracle.chunk_ranges([n], chunk, cmap, k)
+        g = np.concatenate([np.arange(b, e) for b, e in ranges]).astype(np.uint64)
+        s_k = oracle.sigma_eff(1e-3, n, g.size, True)
+        assert abs(s_k - 2e-3) < 1e-18  # sqrt(K) sigma with K = 4 (Sec. 4.1)
+        seeds = np.array([oracle.member_seed(33, 0, k, j) for j in range(P)], np.uint64)
+        coef = np.float32(oracle.step_coef(5e-4, N // K, s_k, oracle.COEF_PAPER))
+        wj = oracle.noise_weights(nid, sign, f_ref[k * (N // K):(k + 1) * (N // K)], P)
+        _, exact, scale = oracle.update_at(g, theta0[g.astype(np.int64)], seeds, wj, coef)
+        assert_update_close(got[g.astype(np.int64)], exact, scale)
+    copes.check()
