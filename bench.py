@@ -67,6 +67,23 @@ def dist_env():
     return rank, world, local
 
 
+def max_over_ranks(value: float, device="cpu") -> float:
+    """The largest of every rank's value (identity when not distributed)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, units_per_step: int, steps: int, seconds: float) -> float:
+    """Whole-job throughput of N independent replicas: every rank processes the full
+    workload, the slowest rank's time counts (weak scaling)."""
+    return world * units_per_step * steps / seconds
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -269,11 +286,7 @@ def main():
             step(s, events)
         end.record()
         torch.cuda.synchronize()
-    ms = start.elapsed_time(end)
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(start.elapsed_time(end), "cuda")
     copes.check()
 
     # end to end through the public API: rewards from pinned host memory each visit,
@@ -292,11 +305,7 @@ def main():
             es.round_robin_visit(arena, subs[k], k, s, cfg, d, r_dev, fitness_out=f_all[k])
         fit_host.copy_(f_all, non_blocking=True)
         torch.cuda.synchronize()
-    e2e_s = time.perf_counter() - t0
-    if world > 1:
-        t = torch.tensor([e2e_s], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks(time.perf_counter() - t0, "cuda")
 
     if rank != 0:
         dist.destroy_process_group() if world > 1 else None
@@ -322,8 +331,8 @@ def main():
     alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12  # Tops/s at the sampled clock
     upd_ops = mean_dk * n_normals_update * alu_ops_per_normal / (per["update"] * 1e-3) / 1e12
     bytes_per_step = d * (wl.n_members * 6 + 6 + 10)
-    value = world * d * args.steps / (ms * 1e-3)
-    e2e = world * d * args.e2e_steps / e2e_s
+    value = job_throughput(world, d, args.steps, ms * 1e-3)
+    e2e = job_throughput(world, d, args.e2e_steps, e2e_s)
     launches = sum(counts.values())
     out = {
         "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
