@@ -286,49 +286,16 @@ __device__ __forceinline__ void noise_weights_to_smem(const UpdateArgs &a, float
 
 template <typename WT, int G, bool COMMIT, bool HI0>
 __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_w,
-                                            const uint32_t (*s_rk)[20], uint64_t b, uint64_t e);
-
-template <typename WT, int G, bool COMMIT>
-__global__ void __launch_bounds__(kThreads) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
-  __shared__ float s_w[COPES_MAX_NOISE];
-  __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
-  noise_weights_to_smem(a, s_w, s_rk);
-  const uint64_t t = blockIdx.x;
-  const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
-  if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
-    if (threadIdx.x == 0) flag_error(kErrTileRange);
-    return;
-  }
-  if ((e >> 34) == 0) update_tile<WT, G, COMMIT, true>(a, s_w, s_rk, b, e);
-  else update_tile<WT, G, COMMIT, false>(a, s_w, s_rk, b, e);
-}
-
-// Members folded into noise weights s_w and round keys s_rk per noise vector; this
-// block's tile [b, e).  HI0 as in elem_values.
-template <typename WT, int G, bool COMMIT, bool HI0>
-__device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_w,
                                             const uint32_t (*s_rk)[20], uint64_t b, uint64_t e) {
   float *__restrict__ master = a.master;
   const uint64_t lo = b & ~3ull;
   const int P = a.n_noise;
   for (uint64_t base = lo + 4ull * threadIdx.x; base < e; base += 4ull * kThreads * G) {
-    float th[G][4], acc[G][4];
-    bool full[G];
+    float acc[G][4];
 #pragma unroll
-    for (int i = 0; i < G; ++i) {
-      const uint64_t g4 = base + 4ull * kThreads * i;
-      full[i] = g4 >= b && g4 + 4 <= e;
-      if (full[i]) {
-        const float4 v = ld_stream_f4(master + g4);
-        th[i][0] = v.x, th[i][1] = v.y, th[i][2] = v.z, th[i][3] = v.w;
-      } else {
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-          th[i][k] = (g4 + k >= b && g4 + k < e) ? master[g4 + k] : 0.0f;
-      }
+    for (int i = 0; i < G; ++i)
 #pragma unroll
       for (int k = 0; k < 4; ++k) acc[i][k] = 0.0f;
-    }
     const uint32_t q_lo = (uint32_t)(base >> 2);  // counter of group 0 (HI0: the whole counter)
     for (int j = 0; j < P; ++j) {
       uint32_t rk[20];
@@ -348,21 +315,21 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
           const uint64_t q = (base >> 2) + kThreads * i;
           philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, w);
         }
-        // scalar Horner here: the packed form needs the coefficient pairs in registers,
-        // which costs this kernel more occupancy than it saves in issue slots
+        // scalar Horner here: measured faster than the packed form in this kernel
         normals4(w, eps);
 #pragma unroll
         for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
       }
     }
+    // theta is read only now, after the noise loop, so it occupies no registers there
 #pragma unroll
     for (int i = 0; i < G; ++i) {
       const uint64_t g4 = base + 4ull * kThreads * i;
       if (g4 >= e) continue;
-      float v[4];
-#pragma unroll
-      for (int k = 0; k < 4; ++k) v[k] = __fmaf_rn(a.coef, acc[i][k], th[i][k]);
-      if (full[i]) {
+      if (g4 >= b && g4 + 4 <= e) {
+        const float4 t = ld_stream_f4(master + g4);
+        float v[4] = {__fmaf_rn(a.coef, acc[i][0], t.x), __fmaf_rn(a.coef, acc[i][1], t.y),
+                      __fmaf_rn(a.coef, acc[i][2], t.z), __fmaf_rn(a.coef, acc[i][3], t.w)};
         st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
         if (COMMIT) WStore<WT>::full(a.w, g4, v);
       } else {
@@ -370,13 +337,31 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
         for (int k = 0; k < 4; ++k) {
           const uint64_t g = g4 + k;
           if (g >= b && g < e) {
-            master[g] = v[k];
-            if (COMMIT) WStore<WT>::one(a.w, g, v[k]);
+            const float v = __fmaf_rn(a.coef, acc[i][k], master[g]);
+            master[g] = v;
+            if (COMMIT) WStore<WT>::one(a.w, g, v);
           }
         }
       }
     }
   }
+}
+
+// One block per tile; the prologue folds the members into noise weights and expands each
+// noise vector's Philox round keys into shared memory.
+template <typename WT, int G, bool COMMIT>
+__global__ void __launch_bounds__(kThreads, 4) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
+  __shared__ float s_w[COPES_MAX_NOISE];
+  __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
+  noise_weights_to_smem(a, s_w, s_rk);
+  const uint64_t t = blockIdx.x;
+  const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
+  if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
+    if (threadIdx.x == 0) flag_error(kErrTileRange);
+    return;
+  }
+  if ((e >> 34) == 0) update_tile<WT, G, COMMIT, true>(a, s_w, s_rk, b, e);
+  else update_tile<WT, G, COMMIT, false>(a, s_w, s_rk, b, e);
 }
 
 template <typename WT, bool COMMIT>
