@@ -170,4 +170,97 @@ __device__ __forceinline__ void st_stream_u2(void *p, uint2 v) {
   __stcs(reinterpret_cast<uint2 *>(p), v);
 }
 
+// ------------------------------------------------------------------------------------
+// Gather-list staging: a block's segment of the int64 index list is brought into shared
+// memory by TMA 1D bulk copies (cp.async.bulk) in chunks, double-buffered on mbarriers,
+// so the next chunk's indices are in flight while the current chunk is processed.
+// Every wait is bounded: after kStageWaitLimit polls the block records kErrStageTimeout,
+// waits (bounded again) for its own copies, and stops.
+constexpr int kStageChunk = 1024;         // indices per chunk (8 KB)
+constexpr int kStageWaitLimit = 1 << 22;  // mbarrier polls before giving up
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p) {
+  return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count));
+}
+
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+// One producer arrival announcing `bytes` of transaction, then the bulk copy itself.
+__device__ __forceinline__ void stage_copy(uint64_t *bar, void *dst, const void *src, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+  if (bytes)
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            smem_addr(dst)),
+        "l"(src), "r"(bytes), "r"(smem_addr(bar))
+        : "memory");
+}
+
+// Polls the barrier's phase `parity` at most kStageWaitLimit times; true once complete.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t *bar, uint32_t parity) {
+  for (int it = 0; it < kStageWaitLimit; ++it) {
+    uint32_t done;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}"
+        : "=r"(done)
+        : "r"(smem_addr(bar)), "r"(parity)
+        : "memory");
+    if (done) return true;
+  }
+  return false;
+}
+
+// Walks the block's segment [s0, s1) of `index` in chunks staged through shared memory;
+// body(const int64_t *chunk_in_smem, int count, uint64_t first_position) runs on every
+// chunk with all threads of the block.  A chunk of odd length copies its even prefix by
+// TMA (sizes must be multiples of 16 bytes) and its last index from global memory into
+// shared memory.  Returns false (after flagging) if a wait timed out.
+template <typename Body, typename Flag>
+__device__ __forceinline__ bool staged_index_segment(const int64_t *index, uint64_t s0, uint64_t s1,
+                                                     int64_t (*buf)[kStageChunk], uint64_t *bar,
+                                                     Flag flag, Body body) {
+  const int n_chunks = (int)((s1 - s0 + kStageChunk - 1) / kStageChunk);
+  auto chunk_count = [&](int c) { return (int)min((uint64_t)kStageChunk, s1 - s0 - (uint64_t)c * kStageChunk); };
+  auto issue = [&](int c) {
+    const int cnt = chunk_count(c);
+    stage_copy(&bar[c & 1], buf[c & 1], index + s0 + (uint64_t)c * kStageChunk, (uint32_t)(cnt & ~1) * 8u);
+  };
+  if (threadIdx.x == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    issue(0);
+    if (n_chunks > 1) issue(1);
+  }
+  for (int c = 0; c < n_chunks; ++c) {
+    const int slot = c & 1;
+    const int cnt = chunk_count(c);
+    if (!mbar_wait_bounded(&bar[slot], (uint32_t)((c >> 1) & 1))) {
+      if (threadIdx.x == 0) flag();
+      // the copy into this block's shared memory may still be in flight: wait once more
+      mbar_wait_bounded(&bar[slot], (uint32_t)((c >> 1) & 1));
+      return false;
+    }
+    if ((cnt & 1) && threadIdx.x == 0) buf[slot][cnt - 1] = index[s0 + (uint64_t)c * kStageChunk + cnt - 1];
+    __syncthreads();
+    body((const int64_t *)buf[slot], cnt, s0 + (uint64_t)c * kStageChunk);
+    __syncthreads();  // every thread is done reading this slot before it is refilled
+    if (threadIdx.x == 0 && c + 2 < n_chunks) {
+      asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+      issue(c + 2);
+    }
+  }
+  return true;
+}
+
 }  // namespace copes

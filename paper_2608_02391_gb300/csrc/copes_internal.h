@@ -78,7 +78,8 @@ __host__ __device__ __forceinline__ void philox4x32_10_rk(uint32_t c0, uint32_t 
 enum : unsigned {
   kErrTileRange = 1u,   // a tile outside [0, n_alloc) or longer than COPES_TILE_MAX
   kErrIndexRange = 2u,  // a gather index outside [0, n_alloc)
-  kErrPartition = 4u    // a partition kernel met an inconsistent workspace
+  kErrPartition = 4u,   // a partition kernel met an inconsistent workspace
+  kErrStageTimeout = 8u // a bulk-copy wait ran past its iteration limit
 };
 
 // ---------------------------------------------------------------- launch arguments

@@ -195,21 +195,27 @@ __global__ void __launch_bounds__(kThreads) elem_tiles_kernel(const ElemArgs a) 
   }
 }
 
+// Gather form: the block's segment of the sorted index list is staged into shared memory
+// chunk by chunk (TMA bulk copies, double-buffered); each thread then handles its indices
+// of the chunk: load theta[g], one Philox word's normal, store w[g] (and theta[g] for init).
 template <int OP, typename WT>
 __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) {
-  constexpr int U = 4;
+  __shared__ __align__(128) int64_t s_idx[2][kStageChunk];
+  __shared__ __align__(8) uint64_t s_bar[2];
+  constexpr int U = kStageChunk / kThreads;
   const uint64_t s0 = (uint64_t)blockIdx.x * kIndexSegment;
   const uint64_t s1 = min(s0 + (uint64_t)kIndexSegment, a.n_index);
   float *__restrict__ master = a.master;
-  for (uint64_t i0 = s0 + threadIdx.x; i0 < s1; i0 += (uint64_t)kThreads * U) {
+  staged_index_segment(a.index, s0, s1, s_idx, s_bar, [] { flag_error(kErrStageTimeout); },
+                       [&](const int64_t *chunk, int cnt, uint64_t) {
     int64_t g[U];
     float th[U];
     bool ok[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
-      const uint64_t i = i0 + (uint64_t)kThreads * u;
-      ok[u] = i < s1;
-      g[u] = ok[u] ? a.index[i] : 0;
+      const int p = threadIdx.x + kThreads * u;
+      ok[u] = p < cnt;
+      g[u] = ok[u] ? chunk[p] : 0;
       if (ok[u] && (g[u] < 0 || (uint64_t)g[u] >= a.n_alloc)) {
         flag_error(kErrIndexRange);
         ok[u] = false;
@@ -226,14 +232,14 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
         uint32_t x[4];
         const uint64_t q = (uint64_t)g[u] >> 2;
         philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, op_tag<OP>(), a.rk, x);
-        const uint32_t s = (uint32_t)g[u] & 3u;
-        const uint32_t wd = s == 0 ? x[0] : (s == 1 ? x[1] : (s == 2 ? x[2] : x[3]));
+        const uint32_t sel = (uint32_t)g[u] & 3u;
+        const uint32_t wd = sel == 0 ? x[0] : (sel == 1 ? x[1] : (sel == 2 ? x[2] : x[3]));
         v = scaled_normal_plus(wd, a.coeffs, OP == kOpPerturb ? th[u] : a.b);
       }
       if (OP == kOpInit) master[g[u]] = v;
       WStore<WT>::one(a.w, (uint64_t)g[u], v);
     }
-  }
+  });
 }
 
 template <int OP, typename WT>
@@ -364,58 +370,64 @@ __global__ void __launch_bounds__(kThreads, 4) update_tiles_kernel(const __grid_
   else update_tile<WT, G, COMMIT, false>(a, s_w, s_rk, b, e);
 }
 
+// Gather form of the update: indices staged through shared memory as in
+// elem_index_kernel; every index regenerates the P normals from its own Philox word.
 template <typename WT, bool COMMIT>
-__global__ void __launch_bounds__(kThreads, 4) update_index_kernel(const __grid_constant__ UpdateArgs a) {
+__global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_constant__ UpdateArgs a) {
   __shared__ float s_w[COPES_MAX_NOISE];
   __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
+  __shared__ __align__(128) int64_t s_idx[2][kStageChunk];
+  __shared__ __align__(8) uint64_t s_bar[2];
   noise_weights_to_smem(a, s_w, s_rk);
   constexpr int U = 2;
   const uint64_t s0 = (uint64_t)blockIdx.x * kIndexSegment;
   const uint64_t s1 = min(s0 + (uint64_t)kIndexSegment, a.n_index);
   float *__restrict__ master = a.master;
   const int P = a.n_noise;
-  for (uint64_t i0 = s0 + threadIdx.x; i0 < s1; i0 += (uint64_t)kThreads * U) {
-    int64_t g[U];
-    float th[U], acc[U];
-    bool ok[U];
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      const uint64_t i = i0 + (uint64_t)kThreads * u;
-      ok[u] = i < s1;
-      g[u] = ok[u] ? a.index[i] : 0;
-      if (ok[u] && (g[u] < 0 || (uint64_t)g[u] >= a.n_alloc)) {
-        flag_error(kErrIndexRange);
-        ok[u] = false;
-      }
-      th[u] = ok[u] ? master[g[u]] : 0.0f;
-      acc[u] = 0.0f;
-    }
-    for (int j = 0; j < P; ++j) {
-      uint32_t rk[20];
-#pragma unroll
-      for (int r = 0; r < 20; r += 4) {
-        const uint4 v = *reinterpret_cast<const uint4 *>(&s_rk[j][r]);
-        rk[r] = v.x, rk[r + 1] = v.y, rk[r + 2] = v.z, rk[r + 3] = v.w;
-      }
-      const float wj = s_w[j];
+  staged_index_segment(a.index, s0, s1, s_idx, s_bar, [] { flag_error(kErrStageTimeout); },
+                       [&](const int64_t *chunk, int cnt, uint64_t) {
+    for (int p0 = threadIdx.x; p0 < cnt; p0 += kThreads * U) {
+      int64_t g[U];
+      float acc[U];
+      bool ok[U];
 #pragma unroll
       for (int u = 0; u < U; ++u) {
-        uint32_t x[4];
-        const uint64_t q = (uint64_t)g[u] >> 2;
-        philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, x);
-        const uint32_t s = (uint32_t)g[u] & 3u;
-        const uint32_t wd = s == 0 ? x[0] : (s == 1 ? x[1] : (s == 2 ? x[2] : x[3]));
-        acc[u] = __fmaf_rn(wj, normal_from_word(wd), acc[u]);
+        const int p = p0 + kThreads * u;
+        ok[u] = p < cnt;
+        g[u] = ok[u] ? chunk[p] : 0;
+        if (ok[u] && (g[u] < 0 || (uint64_t)g[u] >= a.n_alloc)) {
+          flag_error(kErrIndexRange);
+          ok[u] = false;
+        }
+        acc[u] = 0.0f;
+      }
+      for (int j = 0; j < P; ++j) {
+        uint32_t rk[20];
+#pragma unroll
+        for (int r = 0; r < 20; r += 4) {
+          const uint4 v = *reinterpret_cast<const uint4 *>(&s_rk[j][r]);
+          rk[r] = v.x, rk[r + 1] = v.y, rk[r + 2] = v.z, rk[r + 3] = v.w;
+        }
+        const float wj = s_w[j];
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+          uint32_t x[4];
+          const uint64_t q = (uint64_t)g[u] >> 2;
+          philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, x);
+          const uint32_t sel = (uint32_t)g[u] & 3u;
+          const uint32_t wd = sel == 0 ? x[0] : (sel == 1 ? x[1] : (sel == 2 ? x[2] : x[3]));
+          acc[u] = __fmaf_rn(wj, normal_from_word(wd), acc[u]);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        if (!ok[u]) continue;
+        const float v = __fmaf_rn(a.coef, acc[u], master[g[u]]);
+        master[g[u]] = v;
+        if (COMMIT) WStore<WT>::one(a.w, (uint64_t)g[u], v);
       }
     }
-#pragma unroll
-    for (int u = 0; u < U; ++u) {
-      if (!ok[u]) continue;
-      const float v = __fmaf_rn(a.coef, acc[u], th[u]);
-      master[g[u]] = v;
-      if (COMMIT) WStore<WT>::one(a.w, (uint64_t)g[u], v);
-    }
-  }
+  });
 }
 
 template <typename WT, bool COMMIT>
