@@ -353,10 +353,15 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
   }
 }
 
+// Resident blocks per SM of the tile update: 3 x 256 threads leaves 80 registers a thread,
+// enough for G = 4 groups of Philox state, the accumulators and one noise vector's round
+// keys without spilling (measured ~5% faster than 4 blocks at 64 registers).
+constexpr int kUpdateBlocksPerSM = 3;
+
 // One block per tile; the prologue folds the members into noise weights and expands each
 // noise vector's Philox round keys into shared memory.
 template <typename WT, int G, bool COMMIT>
-__global__ void __launch_bounds__(kThreads, 4) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
+__global__ void __launch_bounds__(kThreads, kUpdateBlocksPerSM) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
   __shared__ float s_w[COPES_MAX_NOISE];
   __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
   noise_weights_to_smem(a, s_w, s_rk);
