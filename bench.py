@@ -40,8 +40,8 @@ FALLBACK_HBM_GBS = 6800.0
 # ncu DRAM bytes per element of the dominant kernel (perturb, bf16) from one capture; the
 # figure is dropped (traffic = null) when es_kernels.cu no longer matches the hash it
 # was taken on.
-NCU_TRAFFIC = {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "a3e4ab0eabd4712a",
-               "bytes_per_elem": 5.431, "capture": "profiles/perturb_4b_slice.md"}
+NCU_TRAFFIC = {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "c70a0df3dc6f97c9",
+               "bytes_per_elem": 5.434, "capture": "profiles/perturb_4b_slice.md"}
 
 
 def parse():
