@@ -84,19 +84,30 @@ typedef struct {
 } copes_params;
 
 /* A subspace S (Eq. 7 / Eq. 8: the support of P_k).
- *  TILES:   a device array of n_tiles [begin, end) pairs of uint64 global indices
- *           (tiles[2i], tiles[2i+1]), each of at most COPES_TILE_MAX elements, pairwise
- *           disjoint.  Built by copes_subspace_build (range modes) or
- *           copes_tiles_from_ranges.
- *  INDICES: a device array of n_index int64 global indices, strictly increasing (the
- *           gather form used for hash partitions).  The array must be 16-byte aligned. */
-enum { COPES_SUBSPACE_TILES = 0, COPES_SUBSPACE_INDICES = 1 };
+ *  TILES:       a device array of n_tiles [begin, end) pairs of uint64 global indices
+ *               (tiles[2i], tiles[2i+1]), each of at most COPES_TILE_MAX elements,
+ *               pairwise disjoint.  Built by copes_subspace_build (range modes) or
+ *               copes_tiles_from_ranges.
+ *  INDICES:     a device array of n_index int64 global indices, strictly increasing (the
+ *               gather form used for hash partitions).  The array must be 16-byte aligned.
+ *  HASH_REPLAY: subspace k of the HASH partition (K, seed), with membership recomputed
+ *               from the partition seed inside every kernel instead of read from a list
+ *               (Supp. A.8 "Partition Replay").  Same members as the INDICES list that
+ *               copes_hash_fill writes for (K, seed, k).  Filled by
+ *               copes_hash_replay_subspace; `replay` is a device tensor table it writes. */
+enum { COPES_SUBSPACE_TILES = 0, COPES_SUBSPACE_INDICES = 1, COPES_SUBSPACE_HASH_REPLAY = 2 };
 typedef struct {
   int kind;
-  const uint64_t *tiles; /* TILES: device [2 * n_tiles]  */
+  const uint64_t *tiles;   /* TILES: device [2 * n_tiles]                                */
   uint64_t n_tiles;
-  const int64_t *index;  /* INDICES: device [n_index]    */
+  const int64_t *index;    /* INDICES: device [n_index]                                  */
   uint64_t n_index;
+  const void *replay;      /* HASH_REPLAY: device tensor table (copes_hash_replay_subspace) */
+  uint64_t n_replay_tiles; /* HASH_REPLAY: 16,384-element hash tiles the table covers     */
+  int n_replay_tensors;    /* HASH_REPLAY: entries of the table                           */
+  int K;                   /* HASH_REPLAY: subspaces of the partition, 1 <= K <= COPES_MAX_K */
+  int k;                   /* HASH_REPLAY: this subspace, 0 <= k < K                      */
+  uint64_t seed;           /* HASH_REPLAY: the partition seed                             */
 } copes_subspace;
 
 /* Parameter layout: the model's tensors in order. */
@@ -237,6 +248,22 @@ int copes_hash_fill(const copes_layout_desc *layout, int K, uint64_t seed, void 
 int copes_hash_partition_static(const copes_layout_desc *layout, int K, uint64_t seed,
                                 int64_t *const *lists, const uint64_t *capacity,
                                 uint64_t *counts, cudaStream_t stream);
+
+/* HASH partition by replay (Supp. A.8 "Partition Replay": the partition is kept as its
+ * seed and replayed, not stored as a parameter-level assignment).  Writes the layout's
+ * tensor table (copes_hash_replay_bytes() bytes: 32 per non-empty tensor) into the
+ * device buffer `table` (16-byte aligned, caller-owned; it must outlive every call that
+ * uses *out) with an asynchronous copy on `stream`, and fills *out as the HASH_REPLAY
+ * subspace k of the partition (K, seed).  No list is built: perturb, restore, commit and
+ * update over *out recompute, per 16,384-element tile, each element's bucket
+ * floor(x K / 2^32) (x as in copes_hash_count), gather the tile's members of subspace k
+ * in shared memory and process them.  Results are identical to those over the INDICES
+ * list of (K, seed, k).  The table does not depend on K, seed or k, so the K subspaces of
+ * one partition may share one table. */
+size_t copes_hash_replay_bytes(const copes_layout_desc *layout);
+int copes_hash_replay_subspace(const copes_layout_desc *layout, int K, uint64_t seed, int k,
+                               void *table, size_t table_bytes, cudaStream_t stream,
+                               copes_subspace *out);
 
 /* ------------------------------------------------------------------------- ES steps */
 

@@ -23,7 +23,7 @@ ERR_INVALID_ARG, ERR_ALIGNMENT, ERR_SIZE, ERR_WORKSPACE, ERR_CUDA, ERR_DEVICE_CH
 BF16, FP32 = 0, 1
 TAG_NOISE, TAG_INIT, TAG_PARTITION, TAG_SEED, TAG_CHUNK = 0, 1, 2, 3, 4
 MAX_MEMBERS, MAX_NOISE, MAX_K, TILE_MAX = 256, 256, 64, 1 << 20
-SUBSPACE_TILES, SUBSPACE_INDICES = 0, 1
+SUBSPACE_TILES, SUBSPACE_INDICES, SUBSPACE_HASH_REPLAY = 0, 1, 2
 PART_CONTIGUOUS, PART_TENSOR_GROUPS, PART_HASH, PART_RANDOM_CHUNKS = 0, 1, 2, 3
 SHAPE_NONE, SHAPE_ZSCORE, SHAPE_ZSCORE_GROUPED, SHAPE_CENTERED_RANK = 0, 1, 2, 3
 ONE_SIDED, ANTITHETIC = 0, 1
@@ -47,7 +47,10 @@ class Params(ctypes.Structure):
 
 class Subspace(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int), ("tiles", ctypes.c_void_p), ("n_tiles", ctypes.c_uint64),
-                ("index", ctypes.c_void_p), ("n_index", ctypes.c_uint64)]
+                ("index", ctypes.c_void_p), ("n_index", ctypes.c_uint64),
+                ("replay", ctypes.c_void_p), ("n_replay_tiles", ctypes.c_uint64),
+                ("n_replay_tensors", ctypes.c_int), ("K", ctypes.c_int), ("k", ctypes.c_int),
+                ("seed", ctypes.c_uint64)]
 
 
 class LayoutDesc(ctypes.Structure):
@@ -81,6 +84,8 @@ SIGNATURES = {
     "copes_hash_count": (_I32, [_VP, _I32, _U64, _VP, _SZ, _VP, _VP]),
     "copes_hash_fill": (_I32, [_VP, _I32, _U64, _VP, _SZ, _VP, _VP]),
     "copes_hash_partition_static": (_I32, [_VP, _I32, _U64, _VP, _VP, _VP, _VP]),
+    "copes_hash_replay_bytes": (_SZ, [_VP]),
+    "copes_hash_replay_subspace": (_I32, [_VP, _I32, _U64, _I32, _VP, _SZ, _VP, _VP]),
     "copes_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
     "copes_restore": (_I32, [_VP, _VP, _VP]),
     "copes_context_commit": (_I32, [_VP, _VP, _VP]),
@@ -205,12 +210,16 @@ class Arena:
 
 @dataclass
 class SubspaceHandle:
-    """A subspace: device tiles ([n, 2] int64 holding uint64 bounds) or a device index list."""
+    """A subspace: device tiles ([n, 2] int64 holding uint64 bounds), a device index list, or
+    a hash-replay subspace (tensor = its device tensor table, replay = the filled struct)."""
     kind: int
     tensor: torch.Tensor
     numel: int
+    replay: Optional[Subspace] = None
 
     def struct(self) -> Subspace:
+        if self.kind == SUBSPACE_HASH_REPLAY:
+            return self.replay
         if self.kind == SUBSPACE_TILES:
             return Subspace(SUBSPACE_TILES, self.tensor.data_ptr() if self.tensor.numel() else None,
                             self.tensor.shape[0], None, 0)
@@ -290,6 +299,33 @@ def hash_partition_static(layout: Layout, K: int, seed: int, device="cuda", stre
     _check(L.copes_hash_partition_static(ctypes.byref(layout.desc), K, seed, ptrs, _np_ptr(caps),
                                          _np_ptr(counts), s))
     return [SubspaceHandle(SUBSPACE_INDICES, t[:int(c)], int(c)) for t, c in zip(lists, counts)]
+
+
+def hash_replay_partition(layout: Layout, K: int, seed: int, count: bool = True, device="cuda",
+                          stream=None) -> List[SubspaceHandle]:
+    """copes_hash_replay_subspace for k = 0..K-1: the K subspaces of the hash partition
+    (K, seed) as HASH_REPLAY subspaces sharing one device tensor table; no index list is
+    built.  count=True also counts the members (copes_hash_count on a temporary workspace)
+    so that each handle's numel is known; otherwise numel is -1."""
+    L, s = load(), _stream(stream)
+    nbytes = L.copes_hash_replay_bytes(ctypes.byref(layout.desc))
+    if nbytes == 0:
+        raise CopesError(ERR_INVALID_ARG, "copes_hash_replay_bytes rejected the layout")
+    table = torch.empty(nbytes, dtype=torch.uint8, device=device)
+    counts = np.full(K, -1, np.int64)
+    if count:
+        wbytes = L.copes_hash_workspace_bytes(ctypes.byref(layout.desc), K)
+        ws = torch.empty(wbytes, dtype=torch.uint8, device=device)
+        c = np.zeros(K, np.uint64)
+        _check(L.copes_hash_count(ctypes.byref(layout.desc), K, seed, _ptr(ws), wbytes, _np_ptr(c), s))
+        counts = c.astype(np.int64)
+    handles = []
+    for k in range(K):
+        S = Subspace()
+        _check(L.copes_hash_replay_subspace(ctypes.byref(layout.desc), K, seed, k, _ptr(table), nbytes, s,
+                                            ctypes.byref(S)))
+        handles.append(SubspaceHandle(SUBSPACE_HASH_REPLAY, table, int(counts[k]), S))
+    return handles
 
 
 # -------------------------------------------------------------------------- ES steps

@@ -66,7 +66,30 @@ int check_subspace(const copes_subspace *S, const char *who) {
       return fail(COPES_ERR_SIZE, "%s: index list too long", who);
     return COPES_OK;
   }
+  if (S->kind == COPES_SUBSPACE_HASH_REPLAY) {
+    if (!S->replay) return fail(COPES_ERR_INVALID_ARG, "%s: replay table is NULL", who);
+    if (!aligned(S->replay, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: replay table must be 16-byte aligned", who);
+    if (S->n_replay_tensors < 1 || S->n_replay_tiles < 1)
+      return fail(COPES_ERR_INVALID_ARG, "%s: empty replay table", who);
+    if (S->n_replay_tiles > 0x7FFFFFFFull) return fail(COPES_ERR_SIZE, "%s: more than 2^31-1 hash tiles", who);
+    if (S->K < 1 || S->K > COPES_MAX_K || S->k < 0 || S->k >= S->K)
+      return fail(COPES_ERR_INVALID_ARG, "%s: replay subspace needs 1 <= K <= %d and 0 <= k < K", who,
+                  COPES_MAX_K);
+    return COPES_OK;
+  }
   return fail(COPES_ERR_INVALID_ARG, "%s: unknown subspace kind %d", who, S->kind);
+}
+
+copes::ReplayArgs replay_args(const copes_subspace *S) {
+  copes::ReplayArgs r{};
+  r.table = static_cast<const copes::HashTensor *>(S->replay);
+  r.n_tensors = S->n_replay_tensors;
+  r.n_tiles = S->n_replay_tiles;
+  r.seed_lo = (uint32_t)S->seed;
+  r.seed_hi = (uint32_t)(S->seed >> 32);
+  r.K = S->K;
+  r.k = S->k;
+  return r;
 }
 
 int check_layout(const copes_layout_desc *L, const char *who) {
@@ -136,6 +159,8 @@ int run_elementwise(int op, const copes_params *p, const copes_subspace *S, uint
   // the scale folded into the normal's polynomial: a * eps = x * (a * R(L))
   scaled_coeffs(a_val, a.coeffs);
   copes::philox_round_keys(a.seed_lo, a.seed_hi, a.rk);
+  if (S->kind == COPES_SUBSPACE_HASH_REPLAY)
+    return launch_status(copes::launch_replay_elementwise(op, p->dtype, a, replay_args(S), s), who);
   return launch_status(copes::launch_elementwise(op, S->kind, p->dtype, a, s), who);
 }
 
@@ -184,7 +209,8 @@ int copes_last_error(char *buf, size_t len) {
 int copes_check(cudaStream_t stream) {
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cuda_fail(e, "copes_check");
-  const unsigned bits = copes::read_and_clear_es_errors() | copes::read_and_clear_partition_errors();
+  const unsigned bits = copes::read_and_clear_es_errors() | copes::read_and_clear_partition_errors() |
+                        copes::read_and_clear_replay_errors();
   if ((e = cudaGetLastError()) != cudaSuccess) return cuda_fail(e, "copes_check");
   if (bits)
     return fail(COPES_ERR_DEVICE_CHECK,
@@ -415,6 +441,43 @@ int copes_hash_fill(const copes_layout_desc *layout, int K, uint64_t seed, void 
   return launch_status(e, who);
 }
 
+size_t copes_hash_replay_bytes(const copes_layout_desc *layout) {
+  if (!layout || layout->n_tensors <= 0 || !layout->numel) return 0;
+  return plan_hash(layout, 1).table_bytes;
+}
+
+int copes_hash_replay_subspace(const copes_layout_desc *layout, int K, uint64_t seed, int k,
+                               void *table, size_t table_bytes, cudaStream_t stream,
+                               copes_subspace *out) {
+  const char *who = "copes_hash_replay_subspace";
+  int rc = check_layout(layout, who);
+  if (rc) return rc;
+  if (K < 1 || K > COPES_MAX_K) return fail(COPES_ERR_INVALID_ARG, "%s: K must be in [1, %d]", who, COPES_MAX_K);
+  if (k < 0 || k >= K) return fail(COPES_ERR_INVALID_ARG, "%s: k must be in [0, K)", who);
+  if (!out) return fail(COPES_ERR_INVALID_ARG, "%s: out is NULL", who);
+  const HashPlan plan = plan_hash(layout, K);
+  if (plan.tensors.empty()) return fail(COPES_ERR_SIZE, "%s: the layout has no elements", who);
+  if (plan.n_htiles > 0x7FFFFFFFull) return fail(COPES_ERR_SIZE, "%s: layout too large", who);
+  if (!table || table_bytes < plan.table_bytes)
+    return fail(COPES_ERR_WORKSPACE, "%s: a table of %zu bytes is needed", who, plan.table_bytes);
+  if (!aligned(table, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: table must be 16-byte aligned", who);
+  // Pageable source: the call returns once the data is staged.
+  const cudaError_t e = cudaMemcpyAsync(table, plan.tensors.data(),
+                                        plan.tensors.size() * sizeof(copes::HashTensor),
+                                        cudaMemcpyHostToDevice, stream);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  copes_subspace S{};
+  S.kind = COPES_SUBSPACE_HASH_REPLAY;
+  S.replay = table;
+  S.n_replay_tiles = plan.n_htiles;
+  S.n_replay_tensors = (int)plan.tensors.size();
+  S.K = K;
+  S.k = k;
+  S.seed = seed;
+  *out = S;
+  return COPES_OK;
+}
+
 // ------------------------------------------------------------------------------ ES steps
 int copes_perturb(const copes_params *p, const copes_subspace *S, uint64_t seed,
                   float signed_sigma, cudaStream_t stream) {
@@ -497,6 +560,8 @@ int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
     a.seed_lo[j] = (uint32_t)seeds[j];
     a.seed_hi[j] = (uint32_t)(seeds[j] >> 32);
   }
+  if (S->kind == COPES_SUBSPACE_HASH_REPLAY)
+    return launch_status(copes::launch_replay_update(p->dtype, a, replay_args(S), stream), who);
   return launch_status(copes::launch_update(S->kind, p->dtype, a, stream, 0), who);
 }
 

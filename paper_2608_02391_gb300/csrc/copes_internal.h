@@ -153,6 +153,7 @@ struct HashTensor {
   uint32_t tensor_id;
   uint32_t pad;
 };
+static_assert(sizeof(HashTensor) == 32, "the replay table is documented as 32 bytes per tensor");
 cudaError_t launch_hash_hist(const HashTensor *tensors, int n_tensors, uint64_t n_htiles, int K,
                              uint64_t seed, uint32_t *hist, unsigned long long *totals,
                              cudaStream_t s);
@@ -164,11 +165,26 @@ cudaError_t launch_hash_scatter(const HashTensor *tensors, int n_tensors, uint64
 cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,
                                     cudaStream_t s);
 
+// Partition replay: subspace k of the hash partition (K, seed), recomputed per hash tile
+// from the tensor table (one HashTensor per non-empty tensor, in layout order).
+struct ReplayArgs {
+  const HashTensor *table;
+  int n_tensors;
+  uint64_t n_tiles;  // hash tiles of kHashTile elements covered by the table
+  uint32_t seed_lo, seed_hi;
+  int K, k;
+};
+cudaError_t launch_replay_elementwise(int op, int dtype, const ElemArgs &a, const ReplayArgs &r,
+                                      cudaStream_t s);
+cudaError_t launch_replay_update(int dtype, const UpdateArgs &a, const ReplayArgs &r,
+                                 cudaStream_t s);
+
 // Sets the calling thread's message reported by copes_last_error.
 void set_last_error(const char *message);
 
 // Device error words of each translation unit: read and clear (synchronous).
 unsigned read_and_clear_es_errors();
 unsigned read_and_clear_partition_errors();
+unsigned read_and_clear_replay_errors();
 
 }  // namespace copes

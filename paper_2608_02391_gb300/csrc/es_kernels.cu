@@ -6,6 +6,7 @@
 
 #include "copes_device.cuh"
 #include "copes_internal.h"
+#include "es_common.cuh"
 
 namespace copes {
 
@@ -15,47 +16,6 @@ __device__ __forceinline__ void flag_error(unsigned bit) { atomicOr(&g_es_error,
 
 // ----------------------------------------------------------------- group primitives
 // A "group" is the 4 consecutive global indices 4q .. 4q+3, which share Philox counter q.
-
-template <typename WT>
-struct WStore;
-
-template <>
-struct WStore<__nv_bfloat16> {
-  static __device__ __forceinline__ void full(void *w, uint64_t g, const float v[4]) {
-    uint2 p;
-    p.x = pack_bf16x2(v[0], v[1]);
-    p.y = pack_bf16x2(v[2], v[3]);
-    st_stream_u2(reinterpret_cast<uint16_t *>(w) + g, p);
-  }
-  static __device__ __forceinline__ void one(void *w, uint64_t g, float v) {
-    reinterpret_cast<uint16_t *>(w)[g] = to_bf16_bits(v);
-  }
-};
-
-template <>
-struct WStore<float> {
-  static __device__ __forceinline__ void full(void *w, uint64_t g, const float v[4]) {
-    st_stream_f4(reinterpret_cast<float *>(w) + g, make_float4(v[0], v[1], v[2], v[3]));
-  }
-  static __device__ __forceinline__ void one(void *w, uint64_t g, float v) {
-    reinterpret_cast<float *>(w)[g] = v;
-  }
-};
-
-// scale * eps + b for one word, with scale folded into the coefficients: one fma.
-__device__ __forceinline__ float scaled_normal_plus(uint32_t w, const ScaledCoeffs &k, float b) {
-  float x, r;
-  normal_parts(w, k.central, k.tail, x, r);
-  return __fmaf_rn(r, x, b);
-}
-
-// Noise for the group at 4q under (k0, k1, tag): four normals.
-__device__ __forceinline__ void group_noise(uint64_t q, uint32_t tag, uint32_t k0, uint32_t k1,
-                                            float (&eps)[4]) {
-  uint32_t x[4];
-  philox4x32_10((uint32_t)q, (uint32_t)(q >> 32), 0u, tag, k0, k1, x);
-  normals4(x, eps);
-}
 
 // Noise for a single index g: the one word of its counter that g uses.
 __device__ __forceinline__ float index_noise(uint64_t g, uint32_t tag, uint32_t k0, uint32_t k1) {
@@ -271,25 +231,10 @@ cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, c
 }
 
 // ------------------------------------------------------------------------- update
-// One block per tile.  The prologue folds the members into one weight per noise vector,
-//   w_j = sum_{i : noise(i) = j} sign_i f_i  (member order, fp32),
-// then every thread regenerates all P noise vectors for its groups in registers and
-// accumulates acc = sum_j w_j eps_j (j ascending), theta = fma(coef, acc, theta).
-__device__ __forceinline__ void noise_weights_to_smem(const UpdateArgs &a, float *s_w,
-                                                      uint32_t (*s_rk)[20]) {
-  for (int j = threadIdx.x; j < a.n_noise; j += blockDim.x) {
-    philox_round_keys(a.seed_lo[j], a.seed_hi[j], s_rk[j]);
-    float acc = 0.0f;
-    for (int m = a.noise_ptr[j]; m < a.noise_ptr[j + 1]; ++m) {
-      const int i = a.noise_member[m];
-      const float f = a.fitness[i];
-      acc = __fadd_rn(acc, a.sign[i] > 0 ? f : -f);
-    }
-    s_w[j] = acc;
-  }
-  __syncthreads();
-}
-
+// One block per tile: the prologue (noise_weights_to_smem) folds the members into one
+// weight per noise vector; every thread then regenerates all P noise vectors for its
+// groups in registers and accumulates acc = sum_j w_j eps_j (j ascending),
+// theta = fma(coef, acc, theta).
 template <typename WT, int G, bool COMMIT, bool HI0>
 __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_w,
                                             const uint32_t (*s_rk)[20], uint64_t b, uint64_t e) {

@@ -139,3 +139,42 @@ def test_invalid_arguments_are_rejected_before_any_launch(lib):
     assert lib.copes_subspace_build(ctypes.byref(L.desc), ctypes.byref(spec), 0, 0, None, None, 0,
                                     ctypes.byref(cnt), None) == copes.ERR_SIZE
     assert lib.copes_member_table(7, copes.ANTITHETIC, fake, fake) == copes.ERR_INVALID_ARG
+
+
+def test_hash_replay_arguments_are_rejected_before_any_copy(lib):
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    P = ctypes.c_void_p
+    L = copes.Layout([1000, 0, 2000])
+    assert lib.copes_hash_replay_bytes(ctypes.byref(L.desc)) == 64  # 32 bytes per non-empty tensor
+    assert lib.copes_hash_replay_bytes(None) == 0
+    out = copes.Subspace()
+    for K, k, table, nbytes, code in [(0, 0, fake, 64, copes.ERR_INVALID_ARG),
+                                      (65, 0, fake, 64, copes.ERR_INVALID_ARG),
+                                      (4, 4, fake, 64, copes.ERR_INVALID_ARG),
+                                      (4, -1, fake, 64, copes.ERR_INVALID_ARG),
+                                      (4, 1, None, 64, copes.ERR_WORKSPACE),
+                                      (4, 1, fake, 48, copes.ERR_WORKSPACE),
+                                      (4, 1, fake + 8, 64, copes.ERR_ALIGNMENT)]:
+        assert lib.copes_hash_replay_subspace(ctypes.byref(L.desc), K, 7, k, table, nbytes, None,
+                                              ctypes.byref(out)) == code, (K, k, table, nbytes)
+    assert lib.copes_hash_replay_subspace(ctypes.byref(L.desc), 4, 7, 1, fake, 64, None, None) == \
+        copes.ERR_INVALID_ARG
+    p = copes.Params(fake, fake, 3072, copes.BF16)
+    def replay(**kw):
+        f = dict(kind=copes.SUBSPACE_HASH_REPLAY, replay=fake, n_replay_tiles=2, n_replay_tensors=2, K=4,
+                 k=1, seed=7)
+        f.update(kw)
+        return copes.Subspace(**f)
+    for S, code in [(replay(K=0), copes.ERR_INVALID_ARG), (replay(k=4), copes.ERR_INVALID_ARG),
+                    (replay(replay=None), copes.ERR_INVALID_ARG), (replay(replay=fake + 4), copes.ERR_ALIGNMENT),
+                    (replay(n_replay_tiles=0), copes.ERR_INVALID_ARG),
+                    (replay(n_replay_tiles=1 << 31), copes.ERR_SIZE)]:
+        assert lib.copes_perturb(ctypes.byref(p), ctypes.byref(S), 1, 1e-3, None) == code
+        assert lib.copes_restore(ctypes.byref(p), ctypes.byref(S), None) == code
+    nid = np.array([0, 0], np.int32)
+    sg = np.array([1, -1], np.int8)
+    seeds = np.zeros(1, np.uint64)
+    S = replay(K=65)
+    assert lib.copes_update(ctypes.byref(p), ctypes.byref(S), 2, nid.ctypes.data_as(P), sg.ctypes.data_as(P),
+                            fake, 1, seeds.ctypes.data_as(P), 0.1, 1, None) == copes.ERR_INVALID_ARG

@@ -243,6 +243,52 @@ def test_4b_hash_partition_and_gather_visit(copes):
     copes.check()
 
 
+def test_4b_hash_replay_visit_equals_list_path(copes):
+    """Partition replay at the 4B-hash size: the HASH_REPLAY subspace's visit matches the
+    oracle on sampled members, and its perturb / update equal the INDICES path on the whole
+    arena bit for bit."""
+    w = wl.workload("4b-hash")
+    arena, _ = make_arena(copes, w)
+    tids = list(range(len(w.tensors)))
+    layout = copes.Layout(w.numel, tids)
+    k = 3
+    sub = copes.hash_replay_partition(layout, w.K, w.partition_seed)[k]
+    lst = copes.hash_partition(layout, w.K, w.partition_seed)[k]
+    assert sub.numel == lst.numel
+    nid, sign, P = copes.member_table(w.n_members, copes.ANTITHETIC)
+    seeds = copes.member_seeds(w.base_seed, 0, k, P)
+    # perturb: replay vs list, whole arena
+    copes.perturb(arena, sub, int(seeds[5]), -1e-3)
+    w_replay = arena.w.view(torch.int16).clone()
+    copes.restore(arena, sub)
+    copes.perturb(arena, lst, int(seeds[5]), -1e-3)
+    assert torch.equal(arena.w.view(torch.int16), w_replay)
+    copes.restore(arena, lst)
+    del w_replay
+    # update: replay vs list, whole arena
+    f = torch.linspace(-1.5, 1.5, w.n_members, device="cuda")
+    master0 = arena.master.clone()
+    copes.update(arena, sub, nid, sign, f, seeds, 0.25)
+    m_replay, w_replay = arena.master.clone(), arena.w.view(torch.int16).clone()
+    arena.master.copy_(master0)
+    copes.restore(arena, lst)
+    copes.update(arena, lst, nid, sign, f, seeds, 0.25)
+    assert torch.equal(arena.master.view(torch.int32), m_replay.view(torch.int32))
+    assert torch.equal(arena.w.view(torch.int16), w_replay)
+    del m_replay, w_replay
+    arena.master.copy_(master0)
+    copes.restore(arena, lst)
+    del master0
+    # a visit with the workload's N = 64 on the replay subspace, sampled against the oracle
+    rng = np.random.default_rng(12)
+    pos = np.unique(np.concatenate([[0, 1, lst.numel - 1], rng.integers(0, lst.numel, 4096)]))
+    sample = lst.tensor[torch.from_numpy(pos).cuda()].cpu().numpy()
+    del lst
+    rewards = wl.reward_stream(w, 4)[k]
+    check_visit(copes, arena, sub, sample, w, k, 0, rewards)
+    copes.check()
+
+
 # ----------------------------------------------------------- beyond 2^34 global indices
 def test_counters_beyond_2_34(copes):
     """Tiles past global index 2^34 take the kernels' general counter path; a range
