@@ -14,6 +14,11 @@ update per step, so value = parameters per step x steps / time.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl copes|reference]
 
+`--case 4b-hash` times the non-contiguous workload instead: the same 4B set split by a
+per-element hash into K = 16 subspaces, N = 64 antithetic members, one step = one sweep
+over the 16 subspaces, with the subspaces replayed from the partition seed (default) or
+read from int64 index lists (`--hash-mode lists`).
+
 Prints one JSON line (rank 0).  Under torchrun each rank runs an independent replica on
 its own GPU (the path needs no exchange at this scope), timed with a barrier and the max
 over ranks.
@@ -55,8 +60,11 @@ def parse():
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice"],
-                    help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling")
+    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash"],
+                    help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling; "
+                         "4b-hash: one sweep over the 16 hash subspaces of the 4B set (N=64)")
+    ap.add_argument("--hash-mode", default="replay", choices=["replay", "lists"],
+                    help="4b-hash: subspaces replayed from the partition seed, or int64 index lists")
     return ap.parse_args()
 
 
@@ -215,6 +223,20 @@ def workload_config(wl, args):
 
 
 # -------------------------------------------------------------------------- GPU leg
+def make_arena(copes, torch, wl, layout):
+    """Seeded synthetic weights: fp32 master ~ N(0, init_scale^2), norm tensors 1.0, and
+    w = bf16(master)."""
+    master = torch.empty(layout.d_pad, dtype=torch.float32, device="cuda")
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(wl.init_seed)
+    master.normal_(0.0, wl.init_scale, generator=gen)
+    offs = layout.offsets
+    for t, ten in enumerate(wl.tensors):
+        if ten.kind == "norm":
+            master[int(offs[t]):int(offs[t]) + ten.numel].fill_(1.0)
+    return copes.Arena(master.to(torch.bfloat16), master)
+
+
 def main():
     args = parse()
     from paper_2608_02391_gb300 import workloads
@@ -230,19 +252,12 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     copes.load()
+    if wl.mode == "hash":
+        return run_hash(args, wl, copes, es, torch, rank, world, local)
 
     layout = copes.Layout(wl.numel)
     d = wl.d
-    master = torch.empty(layout.d_pad, dtype=torch.float32, device="cuda")
-    gen = torch.Generator(device="cuda")
-    gen.manual_seed(wl.init_seed)
-    master.normal_(0.0, wl.init_scale, generator=gen)  # seeded synthetic weights
-    offs = layout.offsets
-    for t, ten in enumerate(wl.tensors):
-        if ten.kind == "norm":
-            master[int(offs[t]):int(offs[t]) + ten.numel].fill_(1.0)
-    w = master.to(torch.bfloat16)
-    arena = copes.Arena(w, master)
+    arena = make_arena(copes, torch, wl, layout)
     cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping=wl.shaping)
     total_steps = args.warmup + args.steps + args.e2e_steps
     rewards_host = workloads.reward_stream(wl, total_steps * wl.K)  # [steps*K, N]
@@ -372,6 +387,94 @@ def main():
     print(json.dumps(out), flush=True)
     if world > 1:
         dist.destroy_process_group()
+
+
+def run_hash(args, wl, copes, es, torch, rank, world, local):
+    """The 4B-hash sweep: each of the K = 16 hash subspaces gets one ES iteration with
+    N = 64 members (perturbs, restore, shaping, fused update + commit)."""
+    from paper_2608_02391_gb300 import workloads
+    layout = copes.Layout(wl.numel, list(range(len(wl.tensors))))
+    d = wl.d
+    arena = make_arena(copes, torch, wl, layout)
+    if args.hash_mode == "replay":
+        subs = copes.hash_replay_partition(layout, wl.K, wl.partition_seed)
+    else:
+        subs = copes.hash_partition(layout, wl.K, wl.partition_seed)
+    cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping=wl.shaping)
+    total_steps = args.warmup + args.steps
+    rewards = torch.from_numpy(workloads.reward_stream(wl, total_steps * wl.K)).cuda()
+    fitness = torch.empty(wl.n_members, dtype=torch.float32, device="cuda")
+
+    def step(s, events=None):
+        for k in range(wl.K):
+            es.round_robin_visit(arena, subs[k], k, s, cfg, d, rewards[s * wl.K + k], fitness_out=fitness,
+                                 events=events)
+
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    copes.check()
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    events = {}
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        torch.cuda.synchronize()
+        start.record()
+        for s in range(args.warmup, args.warmup + args.steps):
+            step(s, events)
+        end.record()
+        torch.cuda.synchronize()
+    ms = max_over_ranks(start.elapsed_time(end), "cuda")
+    copes.check()
+    if rank != 0:
+        return
+    per = {name: float(np.mean([a.elapsed_time(b) for a, b in lst])) for name, lst in events.items()}
+    counts = {name: len(lst) for name, lst in events.items()}
+    mean_dk = float(np.mean([s.numel for s in subs]))
+    peaks, peak_src = measured_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    props = torch.cuda.get_device_properties(local)
+    clk = clocks.summary()
+    sm_mhz = clk["sm_mhz"] or float(peaks.get("sm_max_mhz", 2070.0))
+    alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12
+    P = wl.n_members // 2
+    replay = args.hash_mode == "replay"
+    # algorithmic work of one update launch: 28 lane-ops per normal, P normals per member;
+    # replay adds the membership hash of every element (one Philox call = 80 ops per 4)
+    upd_ops = 28.0 * P * mean_dk + (20.0 * d if replay else 0.0)
+    upd_tops = upd_ops / (per["update"] * 1e-3) / 1e12
+    # perturb: 6 B per member (read fp32, write bf16), plus 8 B of index per member for lists
+    pb = (6.0 if replay else 14.0) * mean_dk
+    value = job_throughput(world, d, args.steps, ms * 1e-3)
+    out = {
+        "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": f"4B decoder-shaped bf16 set, fp32 master, K=16 hash subspaces "
+                               f"({args.hash_mode}), N=64 antithetic, one sweep per step",
+                   "params": d, "K": wl.K, "N": wl.n_members, "sigma": wl.sigma, "alpha": wl.alpha,
+                   "shaping": wl.shaping, "hash_mode": args.hash_mode, "partition_seed": wl.partition_seed,
+                   "l2": "inputs larger than L2, no flush"},
+        "roofline": {"bound": "alu", "kernel": "update", "achieved": upd_tops, "peak": alu_peak,
+                     "unit": "Tops/s", "frac": upd_tops / alu_peak, "traffic": None,
+                     "peak_source": "SMs x 128 lanes x sampled SM clock",
+                     "algorithmic_ops_per_launch": upd_ops},
+        "kernels": {
+            "perturb": {"ms": per["perturb"], "launches": counts["perturb"],
+                        "GB/s": pb / (per["perturb"] * 1e-3) / 1e9,
+                        "frac_hbm": pb / (per["perturb"] * 1e-3) / 1e9 / hbm},
+            "restore": {"ms": per["restore"], "launches": counts["restore"]},
+            "update_fused_commit": {"ms": per["update"], "launches": counts["update"], "Tops": upd_tops,
+                                    "frac_alu": upd_tops / alu_peak},
+            "shape": {"ms": per["shape"], "launches": counts["shape"]},
+        },
+        "clocks": clk,
+        "e2e": None,
+        "gpu_launches": sum(counts.values()),
+    }
+    print(json.dumps(out), flush=True)
 
 
 if __name__ == "__main__":

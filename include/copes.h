@@ -251,13 +251,13 @@ int copes_hash_partition_static(const copes_layout_desc *layout, int K, uint64_t
 
 /* HASH partition by replay (Supp. A.8 "Partition Replay": the partition is kept as its
  * seed and replayed, not stored as a parameter-level assignment).  Writes the layout's
- * tensor table (copes_hash_replay_bytes() bytes: 32 per non-empty tensor) into the
- * device buffer `table` (16-byte aligned, caller-owned; it must outlive every call that
- * uses *out) with an asynchronous copy on `stream`, and fills *out as the HASH_REPLAY
- * subspace k of the partition (K, seed).  No list is built: perturb, restore, commit and
- * update over *out recompute, per 16,384-element tile, each element's bucket
- * floor(x K / 2^32) (x as in copes_hash_count), gather the tile's members of subspace k
- * in shared memory and process them.  Results are identical to those over the INDICES
+ * replay table (copes_hash_replay_bytes() bytes: 32 per non-empty tensor, rounded up to
+ * 16, plus 4 per 16,384-element tile, rounded up to 16) into the device buffer `table`
+ * (16-byte aligned, caller-owned; it must outlive every call that uses *out) with
+ * asynchronous copies on `stream`, and fills *out as the HASH_REPLAY subspace k of the
+ * partition (K, seed).  No list is built: perturb, restore, commit and update over *out
+ * recompute, per 16,384-element tile, each element's bucket floor(x K / 2^32) (x as in
+ * copes_hash_count), gather the members of subspace k in shared memory and process them.  Results are identical to those over the INDICES
  * list of (K, seed, k).  The table does not depend on K, seed or k, so the K subspaces of
  * one partition may share one table. */
 size_t copes_hash_replay_bytes(const copes_layout_desc *layout);

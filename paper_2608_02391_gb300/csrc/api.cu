@@ -80,15 +80,26 @@ int check_subspace(const copes_subspace *S, const char *who) {
   return fail(COPES_ERR_INVALID_ARG, "%s: unknown subspace kind %d", who, S->kind);
 }
 
+size_t replay_map_offset(int n_tensors) { return ((size_t)n_tensors * sizeof(copes::HashTensor) + 15) / 16 * 16; }
+
 copes::ReplayArgs replay_args(const copes_subspace *S) {
   copes::ReplayArgs r{};
   r.table = static_cast<const copes::HashTensor *>(S->replay);
+  r.tile_tensor = reinterpret_cast<const uint32_t *>(static_cast<const char *>(S->replay) +
+                                                     replay_map_offset(S->n_replay_tensors));
   r.n_tensors = S->n_replay_tensors;
   r.n_tiles = S->n_replay_tiles;
   r.seed_lo = (uint32_t)S->seed;
   r.seed_hi = (uint32_t)(S->seed >> 32);
   r.K = S->K;
   r.k = S->k;
+  // floor(x K / 2^32) == k  <=>  ceil(k 2^32 / K) <= x < ceil((k + 1) 2^32 / K)
+  const uint64_t lo = (((uint64_t)S->k << 32) + (uint64_t)S->K - 1) / (uint64_t)S->K;
+  const uint64_t hi = (((uint64_t)(S->k + 1) << 32) + (uint64_t)S->K - 1) / (uint64_t)S->K;
+  r.all = S->K == 1;
+  r.lo = (uint32_t)lo;
+  r.width = r.all ? 0u : (uint32_t)(hi - lo);
+  copes::philox_round_keys(r.seed_lo, r.seed_hi, r.rk);
   return r;
 }
 
@@ -443,7 +454,8 @@ int copes_hash_fill(const copes_layout_desc *layout, int K, uint64_t seed, void 
 
 size_t copes_hash_replay_bytes(const copes_layout_desc *layout) {
   if (!layout || layout->n_tensors <= 0 || !layout->numel) return 0;
-  return plan_hash(layout, 1).table_bytes;
+  const HashPlan plan = plan_hash(layout, 1);
+  return plan.table_bytes + round16(plan.n_htiles * 4);
 }
 
 int copes_hash_replay_subspace(const copes_layout_desc *layout, int K, uint64_t seed, int k,
@@ -458,13 +470,21 @@ int copes_hash_replay_subspace(const copes_layout_desc *layout, int K, uint64_t 
   const HashPlan plan = plan_hash(layout, K);
   if (plan.tensors.empty()) return fail(COPES_ERR_SIZE, "%s: the layout has no elements", who);
   if (plan.n_htiles > 0x7FFFFFFFull) return fail(COPES_ERR_SIZE, "%s: layout too large", who);
-  if (!table || table_bytes < plan.table_bytes)
-    return fail(COPES_ERR_WORKSPACE, "%s: a table of %zu bytes is needed", who, plan.table_bytes);
+  const size_t need = plan.table_bytes + round16(plan.n_htiles * 4);
+  if (!table || table_bytes < need)
+    return fail(COPES_ERR_WORKSPACE, "%s: a table of %zu bytes is needed", who, need);
   if (!aligned(table, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: table must be 16-byte aligned", who);
-  // Pageable source: the call returns once the data is staged.
-  const cudaError_t e = cudaMemcpyAsync(table, plan.tensors.data(),
-                                        plan.tensors.size() * sizeof(copes::HashTensor),
-                                        cudaMemcpyHostToDevice, stream);
+  std::vector<uint32_t> tile_tensor(plan.n_htiles);
+  for (size_t t = 0; t < plan.tensors.size(); ++t) {
+    const uint64_t end = t + 1 < plan.tensors.size() ? plan.tensors[t + 1].tile_begin : plan.n_htiles;
+    for (uint64_t i = plan.tensors[t].tile_begin; i < end; ++i) tile_tensor[i] = (uint32_t)t;
+  }
+  // Pageable sources: each copy returns once its data is staged.
+  cudaError_t e = cudaMemcpyAsync(table, plan.tensors.data(), plan.tensors.size() * sizeof(copes::HashTensor),
+                                  cudaMemcpyHostToDevice, stream);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(static_cast<char *>(table) + plan.table_bytes, tile_tensor.data(), plan.n_htiles * 4,
+                        cudaMemcpyHostToDevice, stream);
   if (e != cudaSuccess) return cuda_fail(e, who);
   copes_subspace S{};
   S.kind = COPES_SUBSPACE_HASH_REPLAY;

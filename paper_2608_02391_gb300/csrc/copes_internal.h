@@ -166,13 +166,19 @@ cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uin
                                     cudaStream_t s);
 
 // Partition replay: subspace k of the hash partition (K, seed), recomputed per hash tile
-// from the tensor table (one HashTensor per non-empty tensor, in layout order).
+// from the replay table: one HashTensor per non-empty tensor (layout order), then, from
+// the next 16-byte boundary, the table entry (uint32) of every hash tile.
 struct ReplayArgs {
   const HashTensor *table;
+  const uint32_t *tile_tensor;  // table entry of each hash tile
   int n_tensors;
   uint64_t n_tiles;  // hash tiles of kHashTile elements covered by the table
   uint32_t seed_lo, seed_hi;
   int K, k;
+  // bucket k is the word range [lo, lo + width): lo = ceil(k 2^32 / K); all = (K == 1)
+  uint32_t lo, width;
+  int all;
+  uint32_t rk[20];  // Philox round keys of the partition seed
 };
 cudaError_t launch_replay_elementwise(int op, int dtype, const ElemArgs &a, const ReplayArgs &r,
                                       cudaStream_t s);

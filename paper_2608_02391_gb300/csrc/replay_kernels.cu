@@ -1,15 +1,17 @@
 // Partition replay (Supp. A.8 "Partition Replay"; Eq. 7): the ES kernels over subspace k
 // of the hash partition (K, seed) with membership recomputed from the partition seed, not
-// read from a stored index list.  One block per 16,384-element hash tile of one tensor:
-//  phase 1  every thread hashes its 4-element groups -- one Philox4x32-10 call per group
-//           at counter (e >> 2, tensor id, TAG_PARTITION), bucket floor(x K / 2^32) per
-//           word -- and appends the tile offsets of the members of subspace k to a list
-//           in shared memory (warp-aggregated appends; the list order is arbitrary);
-//  phase 2  the block works through the list exactly as the gather kernels work through
-//           an index list: perturb / restore / commit / init one element per thread, or
-//           the fused update regenerating the P normals of each element.
+// read from a stored index list.  Each block takes 4 consecutive 16,384-element hash
+// tiles; each warp streams through its 2,048-element stretch of every tile (replay_stream):
+//  - it hashes 32 four-element groups at a time -- one Philox4x32-10 call per group at
+//    counter (e >> 2, tensor id, TAG_PARTITION), bucket floor(x K / 2^32) per word -- and
+//    appends the tile offsets of the members of subspace k to its shared-memory buffer;
+//  - whenever the buffer holds a full batch, the warp processes it one member per lane,
+//    exactly as the gather kernels process an index list: perturb / restore / commit /
+//    init, or the fused update regenerating the P normals of each element.
 // Every element's arithmetic is that of the gather path, so the results are identical to
 // those over the INDICES list of (K, seed, k).
+#include <type_traits>
+
 #include "es_common.cuh"
 
 namespace copes {
@@ -18,8 +20,11 @@ __device__ unsigned int g_replay_error = 0;
 
 __device__ __forceinline__ void replay_flag(unsigned bit) { atomicOr(&g_replay_error, bit); }
 
-constexpr int kReplayTile = (int)kHashTile;  // elements per block
-static_assert(kReplayTile % 4 == 0 && kReplayTile <= 65536, "tile offsets are stored as uint16");
+constexpr int kReplayTile = (int)kHashTile;  // elements per hash tile
+constexpr int kReplayTilesPerBlock = 4;      // consecutive hash tiles per block
+static_assert(kReplayTile % 4 == 0 && kReplayTile <= 65536, "tile offsets fit 16 bits");
+constexpr int kReplayWarpGroups = kReplayTile / 4 / (kThreads / 32);  // groups per warp per tile
+constexpr int kReplayIters = kReplayWarpGroups / 32;                  // 32 groups per iteration
 
 struct ReplayTile {
   uint64_t g0;        // global index of the tile's first element
@@ -28,142 +33,188 @@ struct ReplayTile {
   uint32_t tensor_id;
 };
 
-// The tile's tensor and extent.  Thread 0 searches the table; the result is broadcast
-// through shared memory.  A tile outside its tensor or past the arena is skipped and
-// flagged.
-__device__ __forceinline__ void replay_locate(const ReplayArgs &r, uint64_t n_alloc, ReplayTile *s_tile,
-                                              int *s_n) {
-  if (threadIdx.x == 0) {
-    const uint64_t tile = blockIdx.x;
-    int lo = 0, hi = r.n_tensors - 1;  // last entry with tile_begin <= tile
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (r.table[mid].tile_begin <= tile) lo = mid;
-      else hi = mid - 1;
-    }
-    const HashTensor T = r.table[lo];
-    ReplayTile t{};
-    const uint64_t e0 = (tile - T.tile_begin) * (uint64_t)kReplayTile;
-    if (tile < T.tile_begin || e0 >= T.numel) {
-      replay_flag(kErrPartition);
-    } else {
-      t.len = (uint32_t)min((uint64_t)kReplayTile, T.numel - e0);
-      t.g0 = T.offset + e0;
-      t.q0 = e0 >> 2;
-      t.tensor_id = T.tensor_id;
-      if (t.g0 + t.len > n_alloc || (t.g0 & 3ull) != 0) {
-        replay_flag(kErrIndexRange);
-        t.len = 0;
-      }
-    }
-    *s_tile = t;
-    *s_n = 0;
+// Hash tile `tile`: its tensor comes from the table's tile map; every thread reads the
+// same entries (cached broadcasts), so the result is block-uniform.  A tile the table
+// maps outside its tensor or past the arena is skipped and flagged.
+__device__ __forceinline__ ReplayTile replay_tile(const ReplayArgs &r, uint64_t n_alloc, uint64_t tile) {
+  ReplayTile t{};
+  const uint32_t ti = r.tile_tensor[tile];
+  if (ti >= (uint32_t)r.n_tensors) {
+    if (threadIdx.x == 0) replay_flag(kErrPartition);
+    return t;
   }
-  __syncthreads();
+  const HashTensor T = r.table[ti];
+  const uint64_t e0 = (tile - T.tile_begin) * (uint64_t)kReplayTile;
+  if (tile < T.tile_begin || e0 >= T.numel) {
+    if (threadIdx.x == 0) replay_flag(kErrPartition);
+    return t;
+  }
+  const uint32_t len = (uint32_t)min((uint64_t)kReplayTile, T.numel - e0);
+  const uint64_t g0 = T.offset + e0;
+  if (g0 + len > n_alloc || (g0 & 3ull) != 0) {
+    if (threadIdx.x == 0) replay_flag(kErrIndexRange);
+    return t;
+  }
+  t.g0 = g0;
+  t.q0 = e0 >> 2;
+  t.len = len;
+  t.tensor_id = T.tensor_id;
+  return t;
 }
 
-// Phase 1: the tile offsets of the members of subspace r.k, appended to s_list; returns
-// their number.  Every warp runs the same number of iterations, so the full-warp
-// shuffles below see all 32 lanes.
-__device__ __forceinline__ int replay_members(const ReplayArgs &r, const ReplayTile &t,
-                                              uint16_t *s_list, int *s_n) {
-  uint32_t rk[20];
-  philox_round_keys(r.seed_lo, r.seed_hi, rk);
+// Warp-streamed replay over the block's hash tiles.  Each warp owns a 2,048-element
+// stretch of every tile and walks it 32 groups (one per lane) at a time: it hashes the
+// groups, appends the members of subspace r.k to its shared-memory buffer through a shuffle scan of the per-lane counts, and whenever
+// the buffer holds BATCH members it processes them, BATCH / 32 per lane, every lane
+// busy, so the hashing (ALU) interleaves with the members' scattered loads and stores.
+// The warps' leftovers (fewer than BATCH each) are pooled and processed by the whole
+// block at the end.  Every warp runs the same iterations, so full-warp shuffles are safe.
+template <int BATCH, typename Fn, typename Flush>
+__device__ __forceinline__ void replay_stream(const ReplayArgs &r, uint64_t n_alloc, uint32_t *wbuf,
+                                              uint64_t (*s_g0)[kReplayTilesPerBlock], uint32_t *pool,
+                                              int *pool_n, Fn process, Flush flush) {
+  constexpr int U = BATCH / 32;
   const uint32_t lane = threadIdx.x & 31u;
-  const uint32_t n_groups = (t.len + 3u) / 4u;
-  for (uint32_t base = 0; base < n_groups; base += kThreads) {
-    const uint32_t grp = base + threadIdx.x;
-    uint32_t mask = 0;
-    if (grp < n_groups) {
-      const uint64_t q = t.q0 + grp;
-      uint32_t x[4];
-      philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), t.tensor_id, COPES_TAG_PARTITION, rk, x);
+  const uint32_t warp = threadIdx.x >> 5;
+  const uint64_t t_first = (uint64_t)blockIdx.x * kReplayTilesPerBlock;
+  const uint64_t t_end = min(t_first + kReplayTilesPerBlock, r.n_tiles);
+  // buffer entries are (tile within the block) << 16 | (offset within the tile); each warp
+  // keeps the tiles' first global indices in its own row of s_g0
+  uint64_t *wg0 = s_g0[warp];
+  auto global = [&](uint32_t e) { return wg0[e >> 16] + (e & 0xFFFFu); };
+  const uint32_t lt = (1u << lane) - 1u;  // lanes below this one
+  int pending = 0;  // warp-uniform
+  // One iteration: the warp hashes 32 groups (128 elements, one group per lane) and
+  // appends their members with one ballot per word slot; FULL drops the tile-end check.
+  auto iteration = [&](const ReplayTile &t, uint32_t tag, uint32_t q_lo0, uint32_t q_hi, uint32_t e,
+                       auto full) {
+    uint32_t x[4];
+    philox4x32_10_rk(q_lo0 + (e >> 2), q_hi, t.tensor_id, COPES_TAG_PARTITION, r.rk, x);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const uint32_t bucket = (uint32_t)(((uint64_t)x[i] * (uint64_t)r.K) >> 32);
-        if (4u * grp + i < t.len && bucket == (uint32_t)r.k) mask |= 1u << i;
+    for (int i = 0; i < 4; ++i) {
+      // floor(x K / 2^32) == k  <=>  lo <= x < lo + width  (r.lo, r.width from the host)
+      const bool m = (r.all || x[i] - r.lo < r.width) && (decltype(full)::value || e + i < t.len);
+      const uint32_t bal = __ballot_sync(0xffffffffu, m);
+      if (m) wbuf[pending + __popc(bal & lt)] = tag | (e + i);
+      pending += __popc(bal);
+    }
+    __syncwarp();
+    while (pending >= BATCH) {  // take the newest BATCH entries
+      uint64_t g[U];
+      bool ok[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        g[u] = global(wbuf[pending - BATCH + u * 32 + lane]);
+        ok[u] = true;
       }
+      __syncwarp();  // read before the next append overwrites these slots
+      pending -= BATCH;
+      process(g, ok);
     }
-    const int c = __popc(mask);
-    int incl = c;
-#pragma unroll
-    for (int d = 1; d < 32; d <<= 1) {
-      const int y = __shfl_up_sync(0xffffffffu, incl, d);
-      if (lane >= (uint32_t)d) incl += y;
+  };
+  for (uint64_t tile = t_first; tile < t_end; ++tile) {
+    const ReplayTile t = replay_tile(r, n_alloc, tile);
+    const uint32_t tag = (uint32_t)(tile - t_first) << 16;
+    // q0 is a multiple of 4096 and the tile has 4096 groups, so q0 + group never carries
+    // out of 32 bits
+    const uint32_t q_lo0 = (uint32_t)t.q0, q_hi = (uint32_t)(t.q0 >> 32);
+    if (lane == 0) wg0[tile - t_first] = t.g0;
+    __syncwarp();
+    const uint32_t e0 = warp * (4u * kReplayWarpGroups) + 4u * lane;  // this lane's first group
+    if (t.len == (uint32_t)kReplayTile) {
+      for (int it = 0; it < kReplayIters; ++it)
+        iteration(t, tag, q_lo0, q_hi, e0 + 128u * it, std::true_type{});
+    } else if (t.len > 0) {
+      for (int it = 0; it < kReplayIters; ++it)
+        iteration(t, tag, q_lo0, q_hi, e0 + 128u * it, std::false_type{});
     }
-    const int total = __shfl_sync(0xffffffffu, incl, 31);
-    int wbase = 0;
-    if (lane == 31 && total) wbase = atomicAdd(s_n, total);
-    wbase = __shfl_sync(0xffffffffu, wbase, 31);
-    int pos = wbase + incl - c;
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (mask & (1u << i)) s_list[pos++] = (uint16_t)(4u * grp + i);
   }
+  // pool the leftovers and process them with the whole block
+  int at = 0;
+  if (lane == 0 && pending) at = atomicAdd(pool_n, pending);
+  at = __shfl_sync(0xffffffffu, at, 0);
+  for (int p = lane; p < pending; p += 32) pool[at + p] = wbuf[p];
   __syncthreads();
-  return *s_n;
-}
-
-template <int OP>
-constexpr uint32_t replay_tag() { return OP == kOpInit ? COPES_TAG_INIT : COPES_TAG_NOISE; }
-
-// Perturb / restore / commit / init over the members of one hash tile.
-template <int OP, typename WT>
-__global__ void __launch_bounds__(kThreads) replay_elem_kernel(const ElemArgs a, const ReplayArgs r) {
-  __shared__ __align__(16) uint16_t s_list[kReplayTile];
-  __shared__ ReplayTile s_tile;
-  __shared__ int s_n;
-  replay_locate(r, a.n_alloc, &s_tile, &s_n);
-  const ReplayTile t = s_tile;
-  const int n = replay_members(r, t, s_list, &s_n);
-  float *__restrict__ master = a.master;
-  for (int p = threadIdx.x; p < n; p += kThreads) {
-    const uint64_t g = t.g0 + s_list[p];
-    float v;
-    if (OP == kOpRestore) {
-      v = master[g];
-    } else {
-      uint32_t x[4];
-      const uint64_t q = g >> 2;
-      philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, replay_tag<OP>(), a.rk, x);
-      const uint32_t sel = (uint32_t)g & 3u;
-      const uint32_t wd = sel == 0 ? x[0] : (sel == 1 ? x[1] : (sel == 2 ? x[2] : x[3]));
-      v = scaled_normal_plus(wd, a.coeffs, OP == kOpPerturb ? master[g] : a.b);
-      if (OP == kOpInit) master[g] = v;
-    }
-    WStore<WT>::one(a.w, g, v);
-  }
-}
-
-// The fused update over the members of one hash tile.  Dynamic shared memory holds the
-// noise vectors' round keys [P][20], their weights [P] and the member list.
-template <typename WT, bool COMMIT>
-__global__ void __launch_bounds__(kThreads) replay_update_kernel(const __grid_constant__ UpdateArgs a,
-                                                                 const ReplayArgs r) {
-  extern __shared__ __align__(16) unsigned char smem[];
-  auto *s_rk = reinterpret_cast<uint32_t (*)[20]>(smem);
-  float *s_w = reinterpret_cast<float *>(smem + (size_t)a.n_noise * 80);
-  uint16_t *s_list = reinterpret_cast<uint16_t *>(smem + (size_t)a.n_noise * 84);
-  __shared__ ReplayTile s_tile;
-  __shared__ int s_n;
-  noise_weights_to_smem(a, s_w, s_rk);
-  replay_locate(r, a.n_alloc, &s_tile, &s_n);
-  const ReplayTile t = s_tile;
-  const int n = replay_members(r, t, s_list, &s_n);
-  constexpr int U = 2;
-  float *__restrict__ master = a.master;
-  const int P = a.n_noise;
+  const int n = *pool_n;
+  wg0 = s_g0[0];  // every warp recorded the same tiles
   for (int p0 = threadIdx.x; p0 < n; p0 += kThreads * U) {
     uint64_t g[U];
-    float acc[U];
     bool ok[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       const int p = p0 + kThreads * u;
       ok[u] = p < n;
-      g[u] = t.g0 + (ok[u] ? s_list[p] : 0);
-      acc[u] = 0.0f;
+      g[u] = ok[u] ? global(pool[p]) : wg0[0];
     }
+    process(g, ok);
+  }
+  flush();
+}
+
+template <int OP>
+constexpr uint32_t replay_tag() { return OP == kOpInit ? COPES_TAG_INIT : COPES_TAG_NOISE; }
+
+// Perturb / restore / commit / init over the members of the block's hash tiles: four
+// members per lane per batch, their master loads issued together.
+template <int OP, typename WT>
+__global__ void __launch_bounds__(kThreads) replay_elem_kernel(const __grid_constant__ ElemArgs a,
+                                                               const __grid_constant__ ReplayArgs r) {
+  constexpr int BATCH = 128;
+  constexpr int U = BATCH / 32;
+  __shared__ uint32_t s_buf[kThreads / 32][BATCH + 128];
+  __shared__ uint32_t s_pool[(kThreads / 32) * BATCH];
+  __shared__ uint64_t s_g0[kThreads / 32][kReplayTilesPerBlock];
+  __shared__ int s_pool_n;
+  if (threadIdx.x == 0) s_pool_n = 0;
+  __syncthreads();
+  float *__restrict__ master = a.master;
+  replay_stream<BATCH>(r, a.n_alloc, s_buf[threadIdx.x >> 5], s_g0, s_pool, &s_pool_n,
+                       [&](const uint64_t (&g)[U], const bool (&ok)[U]) {
+    float th[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) th[u] = (OP != kOpInit && ok[u]) ? master[g[u]] : 0.0f;
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+      if (!ok[u]) continue;
+      float v;
+      if (OP == kOpRestore) {
+        v = th[u];
+      } else {
+        uint32_t x[4];
+        const uint64_t q = g[u] >> 2;
+        philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, replay_tag<OP>(), a.rk, x);
+        const uint32_t sel = (uint32_t)g[u] & 3u;
+        const uint32_t wd = sel == 0 ? x[0] : (sel == 1 ? x[1] : (sel == 2 ? x[2] : x[3]));
+        v = scaled_normal_plus(wd, a.coeffs, OP == kOpPerturb ? th[u] : a.b);
+        if (OP == kOpInit) master[g[u]] = v;
+      }
+      WStore<WT>::one(a.w, g[u], v);
+    }
+  }, [] {});
+}
+
+// The fused update over the members of the block's hash tiles: two members per lane per
+// batch, each regenerating the P normals of its element.
+template <typename WT, bool COMMIT>
+__global__ void __launch_bounds__(kThreads) replay_update_kernel(const __grid_constant__ UpdateArgs a,
+                                                                 const __grid_constant__ ReplayArgs r) {
+  constexpr int BATCH = 64;
+  constexpr int U = BATCH / 32;
+  __shared__ float s_w[COPES_MAX_NOISE];
+  __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
+  __shared__ uint32_t s_buf[kThreads / 32][BATCH + 128];
+  __shared__ uint32_t s_pool[(kThreads / 32) * BATCH];
+  __shared__ uint64_t s_g0[kThreads / 32][kReplayTilesPerBlock];
+  __shared__ int s_pool_n;
+  if (threadIdx.x == 0) s_pool_n = 0;
+  noise_weights_to_smem(a, s_w, s_rk);  // ends with __syncthreads
+  float *__restrict__ master = a.master;
+  const int P = a.n_noise;
+  replay_stream<BATCH>(r, a.n_alloc, s_buf[threadIdx.x >> 5], s_g0, s_pool, &s_pool_n,
+                       [&](const uint64_t (&g)[U], const bool (&ok)[U]) {
+    float acc[U];
+#pragma unroll
+    for (int u = 0; u < U; ++u) acc[u] = 0.0f;
     for (int j = 0; j < P; ++j) {
       uint32_t rk[20];
 #pragma unroll
@@ -189,13 +240,17 @@ __global__ void __launch_bounds__(kThreads) replay_update_kernel(const __grid_co
       master[g[u]] = v;
       if (COMMIT) WStore<WT>::one(a.w, g[u], v);
     }
-  }
+  }, [] {});
+}
+
+static unsigned replay_blocks(uint64_t n_tiles) {
+  return (unsigned)((n_tiles + kReplayTilesPerBlock - 1) / kReplayTilesPerBlock);
 }
 
 template <int OP, typename WT>
 static cudaError_t launch_replay_elem_typed(const ElemArgs &a, const ReplayArgs &r, cudaStream_t s) {
   if (r.n_tiles == 0) return cudaSuccess;
-  replay_elem_kernel<OP, WT><<<(unsigned)r.n_tiles, kThreads, 0, s>>>(a, r);
+  replay_elem_kernel<OP, WT><<<replay_blocks(r.n_tiles), kThreads, 0, s>>>(a, r);
   return cudaGetLastError();
 }
 
@@ -218,13 +273,7 @@ cudaError_t launch_replay_elementwise(int op, int dtype, const ElemArgs &a, cons
 template <typename WT, bool COMMIT>
 static cudaError_t launch_replay_update_typed(const UpdateArgs &a, const ReplayArgs &r, cudaStream_t s) {
   if (r.n_tiles == 0) return cudaSuccess;
-  const size_t smem = (size_t)a.n_noise * 84 + (size_t)kReplayTile * 2;
-  if (smem > 48 * 1024) {
-    const cudaError_t e = cudaFuncSetAttribute(replay_update_kernel<WT, COMMIT>,
-                                               cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-  }
-  replay_update_kernel<WT, COMMIT><<<(unsigned)r.n_tiles, kThreads, smem, s>>>(a, r);
+  replay_update_kernel<WT, COMMIT><<<replay_blocks(r.n_tiles), kThreads, 0, s>>>(a, r);
   return cudaGetLastError();
 }
 

@@ -146,19 +146,20 @@ def test_hash_replay_arguments_are_rejected_before_any_copy(lib):
     fake = 0x10000  # never dereferenced: every case below fails validation first
     P = ctypes.c_void_p
     L = copes.Layout([1000, 0, 2000])
-    assert lib.copes_hash_replay_bytes(ctypes.byref(L.desc)) == 64  # 32 bytes per non-empty tensor
+    # 32 bytes per non-empty tensor, then 4 per 16,384-element tile (2 tiles), each rounded to 16
+    assert lib.copes_hash_replay_bytes(ctypes.byref(L.desc)) == 80
     assert lib.copes_hash_replay_bytes(None) == 0
     out = copes.Subspace()
-    for K, k, table, nbytes, code in [(0, 0, fake, 64, copes.ERR_INVALID_ARG),
-                                      (65, 0, fake, 64, copes.ERR_INVALID_ARG),
-                                      (4, 4, fake, 64, copes.ERR_INVALID_ARG),
-                                      (4, -1, fake, 64, copes.ERR_INVALID_ARG),
-                                      (4, 1, None, 64, copes.ERR_WORKSPACE),
-                                      (4, 1, fake, 48, copes.ERR_WORKSPACE),
-                                      (4, 1, fake + 8, 64, copes.ERR_ALIGNMENT)]:
+    for K, k, table, nbytes, code in [(0, 0, fake, 80, copes.ERR_INVALID_ARG),
+                                      (65, 0, fake, 80, copes.ERR_INVALID_ARG),
+                                      (4, 4, fake, 80, copes.ERR_INVALID_ARG),
+                                      (4, -1, fake, 80, copes.ERR_INVALID_ARG),
+                                      (4, 1, None, 80, copes.ERR_WORKSPACE),
+                                      (4, 1, fake, 64, copes.ERR_WORKSPACE),
+                                      (4, 1, fake + 8, 80, copes.ERR_ALIGNMENT)]:
         assert lib.copes_hash_replay_subspace(ctypes.byref(L.desc), K, 7, k, table, nbytes, None,
                                               ctypes.byref(out)) == code, (K, k, table, nbytes)
-    assert lib.copes_hash_replay_subspace(ctypes.byref(L.desc), 4, 7, 1, fake, 64, None, None) == \
+    assert lib.copes_hash_replay_subspace(ctypes.byref(L.desc), 4, 7, 1, fake, 80, None, None) == \
         copes.ERR_INVALID_ARG
     p = copes.Params(fake, fake, 3072, copes.BF16)
     def replay(**kw):
