@@ -45,8 +45,8 @@ FALLBACK_HBM_GBS = 6800.0
 # ncu DRAM bytes per element of the dominant kernel (perturb, bf16) from one capture; the
 # figure is dropped (traffic = null) when es_kernels.cu no longer matches the hash it
 # was taken on.
-NCU_TRAFFIC = {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "c70a0df3dc6f97c9",
-               "bytes_per_elem": 5.434, "capture": "profiles/perturb_4b_slice.md"}
+NCU_TRAFFIC = {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "1783d1fcba278162",
+               "bytes_per_elem": 5.431, "capture": "profiles/perturb_4b_slice.md"}
 
 
 def parse():
@@ -60,9 +60,10 @@ def parse():
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash"],
+    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice"],
                     help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling; "
-                         "4b-hash: one sweep over the 16 hash subspaces of the 4B set (N=64)")
+                         "4b-hash: one sweep over the 16 hash subspaces of the 4B set (N=64); "
+                         "4b-hash-slice: the same on 268M parameters, for profiling")
     ap.add_argument("--hash-mode", default="replay", choices=["replay", "lists"],
                     help="4b-hash: subspaces replayed from the partition seed, or int64 index lists")
     return ap.parse_args()
@@ -452,8 +453,9 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
         "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": f"4B decoder-shaped bf16 set, fp32 master, K=16 hash subspaces "
-                               f"({args.hash_mode}), N=64 antithetic, one sweep per step",
+        "config": {"workload": (f"4B decoder-shaped bf16 set, fp32 master" if wl.name == "4b-hash" else
+                                f"{wl.name}: {d} parameters in {len(wl.tensors)} tensors (profiling case)")
+                               + f", K=16 hash subspaces ({args.hash_mode}), N=64 antithetic, one sweep per step",
                    "params": d, "K": wl.K, "N": wl.n_members, "sigma": wl.sigma, "alpha": wl.alpha,
                    "shaping": wl.shaping, "hash_mode": args.hash_mode, "partition_seed": wl.partition_seed,
                    "l2": "inputs larger than L2, no flush"},

@@ -193,6 +193,12 @@ def workload(name: str) -> Workload:
         ts = [Tensor(f"block{i}", 1 << 26, "attn", i) for i in range(4)]
         return Workload("4b-slice", ts, K=4, mode="groups", n_members=32, sigma=1e-3, alpha=5e-4,
                         shaping="zscore", group_of=[0, 1, 2, 3], data_seed=35)
+    if name == "4b-hash-slice":
+        # profiling case of the hash workload: the same K = 16 hash partition and N = 64 on
+        # 4 tensors of 2^26 parameters (1.6 GB resident)
+        ts = [Tensor(f"block{i}", 1 << 26, "attn", i) for i in range(4)]
+        return Workload("4b-hash-slice", ts, K=16, mode="hash", n_members=64, sigma=1e-3, alpha=5e-4,
+                        shaping="zscore", data_seed=36)
     raise KeyError(name)
 
 
