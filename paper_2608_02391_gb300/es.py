@@ -8,6 +8,12 @@ sync_step          one CoPES training step (Algorithm 1): every subspace's N_k =
                    members are evaluated under the same pre-update context, rewards are
                    standardised jointly (Eq. 12) or per subspace (Sec. 4.4 ablation), and
                    all K subspace updates are composed (Eq. 13) before the commit.
+population_visit   round_robin_visit with the population split across the ranks of a
+                   process group, each rank holding a full replica of theta: a rank
+                   evaluates its slice of the members, the N reward scalars are
+                   all-gathered on the host, and every rank applies the same update, so
+                   the replicas stay bit-identical (the paper's population-parallel ES
+                   layout, Sec. 3.3 seed replay: only seeds and scalar rewards travel).
 """
 from __future__ import annotations
 
@@ -120,3 +126,53 @@ def build_subspaces(layout: copes.Layout, mode: str, K: int, group_of: Optional[
         return [copes.subspace_build(layout, copes.PART_RANDOM_CHUNKS, K, k, seed=seed, chunk=chunk,
                                      chunk_map=cmap, tile_size=tile_size) for k in range(K)]
     raise ValueError(mode)
+
+
+# ------------------------------------------------------------- population parallelism
+def member_slice(rank: int, world: int, n_members: int) -> range:
+    """The members rank `rank` evaluates: consecutive blocks of ceil(N / world)."""
+    m = -(-n_members // world)
+    return range(min(rank * m, n_members), min((rank + 1) * m, n_members))
+
+
+def gather_rewards(local: np.ndarray, n_members: int, group=None) -> np.ndarray:
+    """All-gather of the members' rewards over `group` (host tensors; gloo or any backend
+    that gathers CPU tensors).  `local` is a float32 [N] array in which this rank has
+    written the rewards of member_slice(rank, world, N); the result is the full [N] vector,
+    identical on every rank and equal bit for bit to each slice's source values."""
+    import torch.distributed as dist
+    rank, world = dist.get_rank(group), dist.get_world_size(group)
+    m = -(-n_members // world)
+    mine = member_slice(rank, world, n_members)
+    buf = torch.zeros(m, dtype=torch.float32)
+    buf[:len(mine)] = torch.from_numpy(np.ascontiguousarray(local[mine.start:mine.stop], np.float32))
+    parts = [torch.empty(m, dtype=torch.float32) for _ in range(world)]
+    dist.all_gather(parts, buf, group=group)
+    return torch.cat(parts)[:n_members].numpy()
+
+
+def population_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iteration: int,
+                     cfg: ESConfig, d: int, evaluate: Callable[[int], float], group=None,
+                     fitness_out: Optional[torch.Tensor] = None) -> torch.Tensor:
+    """One ES iteration on subspace k, population-parallel over the ranks of `group`.
+    Every rank holds the same theta; rank r evaluates members member_slice(r, R, N):
+    perturb, evaluate(i) -> reward (host float) while the perturbation is live, and
+    restores S afterwards.  The rewards are all-gathered, then every rank shapes the same
+    vector and applies the same fused update + commit, so the replicas stay identical."""
+    import torch.distributed as dist
+    rank, world = dist.get_rank(group), dist.get_world_size(group)
+    N = cfg.n_members
+    nid, sign, P = copes.member_table(N, cfg.pairing)
+    seeds = copes.member_seeds(cfg.base_seed, iteration, k, P)
+    s_k = sigma_k(cfg, d, sub.numel)
+    local = np.zeros(N, np.float32)
+    for i in member_slice(rank, world, N):
+        copes.perturb(arena, sub, int(seeds[nid[i]]), float(sign[i]) * s_k)
+        local[i] = np.float32(evaluate(i))
+    copes.restore(arena, sub)
+    rewards = torch.from_numpy(gather_rewards(local, N, group)).to(arena.w.device)
+    f = fitness_out if fitness_out is not None else torch.empty_like(rewards)
+    copes.shape_fitness(rewards, cfg.shaping, out=f)
+    coef = copes.step_coef(cfg.alpha, N, s_k, cfg.convention)
+    copes.update(arena, sub, nid, sign, f, seeds, coef, fuse_commit=True)
+    return f

@@ -1,0 +1,93 @@
+"""Population-parallel ES on the GPU: two ranks (processes) with full replicas of theta
+split the members of every visit, exchange the reward scalars over gloo, and apply the
+same update.  After a cycle over the K subspaces their masters and working weights are
+bit-identical, and equal to a single process running the whole population.  The ranks'
+kernels never wait on one another: the only synchronisation is the host all-gather."""
+import hashlib
+import os
+import socket
+import sys
+
+import numpy as np
+import pytest
+import torch.multiprocessing as mp
+
+pytestmark = pytest.mark.gpu
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+N_PARAMS = 1 << 20
+K, N = 4, 16
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _setup():
+    import torch
+    sys.path.insert(0, ROOT)
+    from paper_2608_02391_gb300 import copes, es
+    copes.load()
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(0)
+    master = torch.empty(N_PARAMS, device="cuda").normal_(0.0, 0.02, generator=gen)
+    arena = copes.Arena(master.to(torch.bfloat16), master)
+    c = torch.empty(N_PARAMS, device="cuda").normal_(0.0, 1.0, generator=gen)
+    layout = copes.Layout([N_PARAMS])
+    subs = es.build_subspaces(layout, "contiguous", K, tile_size=4096)
+    cfg = es.ESConfig(n_members=N, sigma=1e-3, alpha=5e-4, shaping="zscore")
+    return torch, copes, es, arena, c, subs, cfg
+
+
+def _digest(torch, arena):
+    """Hash of the master's and the working weights' bits."""
+    return hashlib.sha256(arena.master.cpu().numpy().tobytes() +
+                          arena.w.view(torch.int16).cpu().numpy().tobytes()).hexdigest()
+
+
+def _worker(rank, world, port, out):
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        torch, copes, es, arena, c, subs, cfg = _setup()
+
+        def evaluate(i):  # the reward of the live perturbation: a linear objective
+            return float((c * arena.w.float()).sum().item())
+
+        for k in range(K):
+            es.population_visit(arena, subs[k], k, 0, cfg, N_PARAMS, evaluate)
+        copes.check()
+        digest = _digest(torch, arena)
+        ref = None
+        if rank == 0:  # the same cycle in one process, whole population
+            torch, copes, es, arena1, c1, subs1, cfg1 = _setup()
+            for k in range(K):
+                rewards = torch.empty(N, device="cuda")
+
+                def ev(i, rewards=rewards):
+                    rewards[i] = (c1 * arena1.w.float()).sum()
+                es.round_robin_visit(arena1, subs1[k], k, 0, cfg1, N_PARAMS, rewards, evaluate=ev)
+            copes.check()
+            ref = _digest(torch, arena1)
+        out.put((rank, digest, ref))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_two_ranks_stay_bit_identical_and_match_one_process():
+    ctx = mp.get_context("spawn")
+    out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    res = sorted(out.get(timeout=600) for _ in procs)
+    for p in procs:
+        p.join(timeout=120)
+        assert p.exitcode == 0
+    (r0, d0, ref), (r1, d1, _) = res
+    assert d0 == d1
+    assert d0 == ref
