@@ -14,6 +14,9 @@ update per step, so value = parameters per step x steps / time.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl copes|reference]
 
+`--case 4b-backup` times the 4B step in the CPU weight backup mode: bf16 weights on the
+GPU, the context in pinned host memory, no fp32 master.
+
 `--case 4b-hash` times the non-contiguous workload instead: the same 4B set split by a
 per-element hash into K = 16 subspaces, N = 64 antithetic members, one step = one sweep
 over the 16 subspaces, with the subspaces replayed from the partition seed (default) or
@@ -60,10 +63,11 @@ def parse():
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice"],
+    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice", "4b-backup"],
                     help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling; "
                          "4b-hash: one sweep over the 16 hash subspaces of the 4B set (N=64); "
-                         "4b-hash-slice: the same on 268M parameters, for profiling")
+                         "4b-hash-slice: the same on 268M parameters, for profiling; "
+                         "4b-backup: the 4B step in the CPU weight backup mode (no fp32 master)")
     ap.add_argument("--hash-mode", default="replay", choices=["replay", "lists"],
                     help="4b-hash: subspaces replayed from the partition seed, or int64 index lists")
     return ap.parse_args()
@@ -241,7 +245,7 @@ def make_arena(copes, torch, wl, layout):
 def main():
     args = parse()
     from paper_2608_02391_gb300 import workloads
-    wl = workloads.workload(args.case)
+    wl = workloads.workload("4b" if args.case == "4b-backup" else args.case)
     if args.impl == "reference":
         return run_reference(args, wl)
 
@@ -255,6 +259,8 @@ def main():
     copes.load()
     if wl.mode == "hash":
         return run_hash(args, wl, copes, es, torch, rank, world, local)
+    if args.case == "4b-backup":
+        return run_backup(args, wl, copes, es, torch, rank, world, local)
 
     layout = copes.Layout(wl.numel)
     d = wl.d
@@ -473,6 +479,101 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
             "shape": {"ms": per["shape"], "launches": counts["shape"]},
         },
         "clocks": clk,
+        "e2e": None,
+        "gpu_launches": sum(counts.values()),
+    }
+    print(json.dumps(out), flush=True)
+
+
+def host_link_gbs(torch, nbytes=1 << 30, reps=5):
+    """Measured copy bandwidth of the host link: pinned host -> device and device -> pinned
+    host, cudaMemcpyAsync of 1 GiB, best of `reps`."""
+    h = torch.empty(nbytes, dtype=torch.uint8).pin_memory()
+    dv = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    out = {}
+    for name, (dst, src) in {"h2d": (dv, h), "d2h": (h, dv)}.items():
+        best = 0.0
+        for _ in range(reps):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            dst.copy_(src, non_blocking=True)
+            b.record()
+            torch.cuda.synchronize()
+            best = max(best, nbytes / (a.elapsed_time(b) * 1e-3) / 1e9)
+        out[name] = best
+    return out
+
+
+def run_backup(args, wl, copes, es, torch, rank, world, local):
+    """The 4B step in the CPU weight backup mode: per visit, save the subspace's context to
+    pinned host memory, 32 perturbs from it, restore, shaping and the update (which
+    writes the new context to both copies)."""
+    from paper_2608_02391_gb300 import workloads
+    layout = copes.Layout(wl.numel)
+    d = wl.d
+    full = make_arena(copes, torch, wl, layout)
+    w = full.w
+    del full
+    backup = torch.empty(w.numel(), dtype=torch.bfloat16).pin_memory()
+    arena = copes.BackupArena(w, backup)
+    subs = es.build_subspaces(layout, "groups", wl.K, group_of=wl.group_of, tile_size=args.tile)
+    for sub in subs:
+        copes.backup_save(arena, sub)
+    cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping=wl.shaping)
+    total = args.warmup + args.steps
+    rewards = torch.from_numpy(workloads.reward_stream(wl, total * wl.K)).cuda()
+    fitness = torch.empty(wl.n_members, dtype=torch.float32, device="cuda")
+
+    def step(s, events=None):
+        for k in range(wl.K):
+            es.backup_visit(arena, subs[k], k, s, cfg, d, rewards[s * wl.K + k], fitness_out=fitness,
+                            events=events)
+
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    copes.check()
+    events = {}
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        torch.cuda.synchronize()
+        start.record()
+        for s in range(args.warmup, args.warmup + args.steps):
+            step(s, events)
+        end.record()
+        torch.cuda.synchronize()
+    ms = max_over_ranks(start.elapsed_time(end), "cuda")
+    copes.check()
+    if rank != 0:
+        return
+    link = host_link_gbs(torch)
+    per = {name: float(np.mean([a.elapsed_time(b) for a, b in lst])) for name, lst in events.items()}
+    counts = {name: len(lst) for name, lst in events.items()}
+    mean_dk = float(np.mean([s.numel for s in subs]))
+    # bytes crossing the host link per launch (bf16 = 2 B per element)
+    host_bytes = {"save": 2.0, "perturb": 2.0, "restore": 2.0, "update": 4.0}
+    kern = {}
+    for name, hb in host_bytes.items():
+        gbs = hb * mean_dk / (per[name] * 1e-3) / 1e9
+        ref = link["d2h"] if name == "save" else link["h2d"]
+        kern[name] = {"ms": per[name], "launches": counts[name], "host_link_GB/s": gbs, "frac_link": gbs / ref}
+    kern["shape"] = {"ms": per["shape"], "launches": counts["shape"]}
+    value = job_throughput(world, d, args.steps, ms * 1e-3)
+    p_gbs = kern["perturb"]["host_link_GB/s"]
+    out = {
+        "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "4B decoder-shaped bf16 set, K=8 layer blocks, N=32 antithetic, CPU weight "
+                               "backup mode (bf16 context in pinned host memory, no fp32 master)",
+                   "params": d, "K": wl.K, "N": wl.n_members, "tile": args.tile,
+                   "l2": "inputs larger than L2, no flush"},
+        "roofline": {"bound": "host_link", "kernel": "perturb", "achieved": p_gbs, "peak": link["h2d"],
+                     "unit": "GB/s", "frac": p_gbs / link["h2d"], "traffic": None,
+                     "peak_source": "measured pinned host->device cudaMemcpyAsync of 1 GiB"},
+        "host_link_measured_GB/s": link,
+        "kernels": kern,
+        "clocks": clocks.summary(),
         "e2e": None,
         "gpu_launches": sum(counts.values()),
     }

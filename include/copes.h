@@ -306,6 +306,43 @@ int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
 int copes_init_normal(const copes_params *p, const copes_subspace *S, uint64_t seed,
                       float mean, float scale, cudaStream_t stream);
 
+/* ----------------------------------------------------------- CPU weight backup mode */
+
+/* CPU weight backup (Supp. A.8 "CPU Weight Backup"): for a GPU on which an fp32 master
+ * does not fit, the working weights stay bf16 in HBM and the pre-perturbation weights
+ * (the shared context) are kept as a bf16 copy in pinned host memory, which the kernels
+ * read and write directly (on GB300 across NVLink-C2C).  Perturbations are computed from
+ * the backup, never from the live weights, so every member is evaluated from the same
+ * pre-update model and perturb stays idempotent; restore copies the backup back, with no
+ * subtraction of replayed noise.
+ *  w:       device bf16 [n_alloc], the weights the model reads;
+ *  backup:  host bf16 [n_alloc] in page-locked memory (cudaHostAlloc / cudaHostRegister,
+ *           or torch's pin_memory()); any other pointer gives COPES_ERR_INVALID_ARG.
+ * Only TILES subspaces are supported (COPES_ERR_UNSUPPORTED otherwise).  Both buffers are
+ * indexed by the global index g, like w and master in copes_params. */
+typedef struct {
+  void *w;           /* device bf16 [n_alloc]                 */
+  uint16_t *backup;  /* pinned host bf16 [n_alloc]            */
+  uint64_t n_alloc;
+} copes_backup_params;
+
+/* backup[g] = w[g] for g in S (the context is saved before the members are evaluated). */
+int copes_backup_save(const copes_backup_params *p, const copes_subspace *S, cudaStream_t stream);
+
+/* Perturb from the backup (Eq. 8): w[g] = round(fma(signed_sigma, eps_seed[g], backup[g])). */
+int copes_backup_perturb(const copes_backup_params *p, const copes_subspace *S, uint64_t seed,
+                         float signed_sigma, cudaStream_t stream);
+
+/* Restore (Supp. A.8): w[g] = backup[g], bit-exact. */
+int copes_backup_restore(const copes_backup_params *p, const copes_subspace *S, cudaStream_t stream);
+
+/* Update from the backup (Eq. 6, Eq. 13), with the arguments of copes_update:
+ *   t = fma(coef, acc, backup[g]) in fp32,  w[g] = backup[g] = round(t),
+ * so the new context is both published to the model and saved as the next backup. */
+int copes_backup_update(const copes_backup_params *p, const copes_subspace *S, int n_members,
+                        const int32_t *noise_id, const int8_t *sign, const float *fitness,
+                        int n_noise, const uint64_t *seeds, float coef, cudaStream_t stream);
+
 /* ------------------------------------------------------------------- debug exports */
 
 /* Philox words for counters q0 .. q0+n-1 with (aux, tag): out is device uint32 [4n]. */

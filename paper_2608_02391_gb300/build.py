@@ -15,8 +15,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 LIB = os.path.join(HERE, "libcopes.so")
 BUILD_DIR = os.path.join(HERE, "_build")
-SOURCES = ["api.cu", "es_kernels.cu", "replay_kernels.cu", "shape_kernels.cu", "partition_kernels.cu",
-           "hash_static.cu"]
+SOURCES = ["api.cu", "es_kernels.cu", "replay_kernels.cu", "backup_kernels.cu", "shape_kernels.cu",
+           "partition_kernels.cu", "hash_static.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-Xptxas", "-warn-spills"]

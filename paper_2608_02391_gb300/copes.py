@@ -53,6 +53,10 @@ class Subspace(ctypes.Structure):
                 ("seed", ctypes.c_uint64)]
 
 
+class BackupParams(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("backup", ctypes.c_void_p), ("n_alloc", ctypes.c_uint64)]
+
+
 class LayoutDesc(ctypes.Structure):
     _fields_ = [("n_tensors", ctypes.c_int), ("numel", ctypes.c_void_p), ("tensor_id", ctypes.c_void_p)]
 
@@ -92,6 +96,10 @@ SIGNATURES = {
     "copes_shape_fitness": (_I32, [_VP, _I32, _VP, _I32, _VP, _VP]),
     "copes_update": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _F32, _I32, _VP]),
     "copes_init_normal": (_I32, [_VP, _VP, _U64, _F32, _F32, _VP]),
+    "copes_backup_save": (_I32, [_VP, _VP, _VP]),
+    "copes_backup_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
+    "copes_backup_restore": (_I32, [_VP, _VP, _VP]),
+    "copes_backup_update": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _F32, _VP]),
     "copes_debug_philox": (_I32, [_U64, _U64, _U64, _U32, _U32, _VP, _VP]),
     "copes_debug_normals": (_I32, [_U64, _U32, _U64, _U64, _VP, _VP]),
     "copes_debug_transform": (_I32, [_VP, _U64, _VP, _VP]),
@@ -390,3 +398,47 @@ def debug_transform(words: torch.Tensor, stream=None) -> torch.Tensor:
     out = torch.empty(words.numel(), dtype=torch.float32, device=words.device)
     _check(load().copes_debug_transform(_ptr(words), words.numel(), _ptr(out), _stream(stream)))
     return out
+
+
+# ------------------------------------------------------------------ CPU weight backup
+class BackupArena:
+    """CPU weight backup mode: bf16 working weights on the device and the shared context as
+    a bf16 copy in page-locked host memory (no fp32 master)."""
+
+    def __init__(self, w: torch.Tensor, backup: torch.Tensor):
+        assert w.is_cuda and w.dtype == torch.bfloat16 and w.is_contiguous()
+        assert backup.dtype == torch.bfloat16 and not backup.is_cuda and backup.numel() == w.numel()
+        self.w, self.backup = w, backup
+        self.params = BackupParams(w.data_ptr(), backup.data_ptr(), w.numel())
+
+    @classmethod
+    def empty(cls, n: int, device="cuda"):
+        return cls(torch.empty(n, dtype=torch.bfloat16, device=device),
+                   torch.empty(n, dtype=torch.bfloat16).pin_memory())
+
+
+def backup_save(arena: BackupArena, sub: SubspaceHandle, stream=None) -> None:
+    S = sub.struct()
+    _check(load().copes_backup_save(ctypes.byref(arena.params), ctypes.byref(S), _stream(stream)))
+
+
+def backup_perturb(arena: BackupArena, sub: SubspaceHandle, seed: int, signed_sigma: float, stream=None) -> None:
+    S = sub.struct()
+    _check(load().copes_backup_perturb(ctypes.byref(arena.params), ctypes.byref(S), seed, signed_sigma,
+                                       _stream(stream)))
+
+
+def backup_restore(arena: BackupArena, sub: SubspaceHandle, stream=None) -> None:
+    S = sub.struct()
+    _check(load().copes_backup_restore(ctypes.byref(arena.params), ctypes.byref(S), _stream(stream)))
+
+
+def backup_update(arena: BackupArena, sub: SubspaceHandle, noise_id: np.ndarray, sign: np.ndarray,
+                  fitness: torch.Tensor, seeds: np.ndarray, coef: float, stream=None) -> None:
+    nid = np.ascontiguousarray(noise_id, np.int32)
+    sg = np.ascontiguousarray(sign, np.int8)
+    sd = np.ascontiguousarray(seeds, np.uint64)
+    assert fitness.dtype == torch.float32 and fitness.is_cuda and fitness.numel() == nid.size
+    S = sub.struct()
+    _check(load().copes_backup_update(ctypes.byref(arena.params), ctypes.byref(S), nid.size, _np_ptr(nid),
+                                      _np_ptr(sg), _ptr(fitness), sd.size, _np_ptr(sd), coef, _stream(stream)))

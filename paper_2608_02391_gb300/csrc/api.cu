@@ -221,7 +221,7 @@ int copes_check(cudaStream_t stream) {
   cudaError_t e = cudaStreamSynchronize(stream);
   if (e != cudaSuccess) return cuda_fail(e, "copes_check");
   const unsigned bits = copes::read_and_clear_es_errors() | copes::read_and_clear_partition_errors() |
-                        copes::read_and_clear_replay_errors();
+                        copes::read_and_clear_replay_errors() | copes::read_and_clear_backup_errors();
   if ((e = cudaGetLastError()) != cudaSuccess) return cuda_fail(e, "copes_check");
   if (bits)
     return fail(COPES_ERR_DEVICE_CHECK,
@@ -532,13 +532,13 @@ int copes_shape_fitness(const float *rewards, int n, const int32_t *group, int m
   return launch_status(copes::launch_shape(rewards, n, group, mode, fitness, stream), who);
 }
 
-int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
-                 const int32_t *noise_id, const int8_t *sign, const float *fitness, int n_noise,
-                 const uint64_t *seeds, float coef, int fuse_commit, cudaStream_t stream) {
-  const char *who = "copes_update";
-  int rc = check_params(p, who);
-  if (rc) return rc;
-  if ((rc = check_subspace(S, who))) return rc;
+namespace {
+
+// The update's member arguments: checks them and fills the noise weights' member table
+// (CSR, member order kept within each noise id) and the seeds into `a`.
+int fill_update_members(UpdateArgs &a, int n_members, const int32_t *noise_id, const int8_t *sign,
+                        const float *fitness, int n_noise, const uint64_t *seeds, float coef,
+                        const char *who) {
   if (n_members < 1 || n_members > COPES_MAX_MEMBERS)
     return fail(COPES_ERR_SIZE, "%s: n_members must be in [1, %d]", who, COPES_MAX_MEMBERS);
   if (n_noise < 1 || n_noise > COPES_MAX_NOISE)
@@ -546,23 +546,10 @@ int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
   if (!noise_id || !sign || !fitness || !seeds)
     return fail(COPES_ERR_INVALID_ARG, "%s: noise_id, sign, fitness and seeds are required", who);
   if (!isfinite(coef)) return fail(COPES_ERR_INVALID_ARG, "%s: coef is not finite", who);
-  UpdateArgs a{};
-  a.w = p->w;
-  a.master = p->master;
-  a.n_alloc = p->n_alloc;
-  if (S->kind == COPES_SUBSPACE_TILES) {
-    a.tiles = S->tiles;
-    a.n_tiles = S->n_tiles;
-  } else {
-    a.index = S->index;
-    a.n_index = S->n_index;
-  }
   a.fitness = fitness;
   a.coef = coef;
   a.n_members = n_members;
   a.n_noise = n_noise;
-  a.fuse_commit = fuse_commit ? 1 : 0;
-  // members grouped by noise vector (CSR, member order kept within each noise id)
   std::vector<int> count(n_noise + 1, 0);
   for (int i = 0; i < n_members; ++i) {
     if (noise_id[i] < 0 || noise_id[i] >= n_noise)
@@ -580,9 +567,104 @@ int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
     a.seed_lo[j] = (uint32_t)seeds[j];
     a.seed_hi[j] = (uint32_t)(seeds[j] >> 32);
   }
+  return COPES_OK;
+}
+
+// Backup mode: checks the arguments and resolves the device address of the pinned backup.
+int check_backup(const copes_backup_params *p, const copes_subspace *S, const char *who,
+                 uint16_t **backup_dev) {
+  if (!p) return fail(COPES_ERR_INVALID_ARG, "%s: params is NULL", who);
+  if (!p->w || !p->backup) return fail(COPES_ERR_INVALID_ARG, "%s: w or backup is NULL", who);
+  if (!aligned(p->w, 16) || !aligned(p->backup, 16))
+    return fail(COPES_ERR_ALIGNMENT, "%s: w and backup must be 16-byte aligned", who);
+  if (p->n_alloc == 0) return fail(COPES_ERR_SIZE, "%s: n_alloc is 0", who);
+  int rc = check_subspace(S, who);
+  if (rc) return rc;
+  if (S->kind != COPES_SUBSPACE_TILES)
+    return fail(COPES_ERR_UNSUPPORTED, "%s: the backup mode takes TILES subspaces only", who);
+  cudaPointerAttributes attr{};
+  const cudaError_t e = cudaPointerGetAttributes(&attr, p->backup);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  if (attr.type != cudaMemoryTypeHost || !attr.devicePointer)
+    return fail(COPES_ERR_INVALID_ARG, "%s: backup must be page-locked host memory", who);
+  *backup_dev = static_cast<uint16_t *>(attr.devicePointer);
+  return COPES_OK;
+}
+
+int run_backup_elementwise(int op, const copes_backup_params *p, const copes_subspace *S, uint64_t seed,
+                           float sigma, cudaStream_t s, const char *who) {
+  uint16_t *dev = nullptr;
+  int rc = check_backup(p, S, who, &dev);
+  if (rc) return rc;
+  ElemArgs a{};
+  a.w = p->w;
+  a.n_alloc = p->n_alloc;
+  a.tiles = S->tiles;
+  a.n_tiles = S->n_tiles;
+  a.seed_lo = (uint32_t)seed;
+  a.seed_hi = (uint32_t)(seed >> 32);
+  a.a = sigma;
+  scaled_coeffs(sigma, a.coeffs);
+  copes::philox_round_keys(a.seed_lo, a.seed_hi, a.rk);
+  return launch_status(copes::launch_backup_elementwise(op, a, dev, s), who);
+}
+
+}  // namespace
+
+int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
+                 const int32_t *noise_id, const int8_t *sign, const float *fitness, int n_noise,
+                 const uint64_t *seeds, float coef, int fuse_commit, cudaStream_t stream) {
+  const char *who = "copes_update";
+  int rc = check_params(p, who);
+  if (rc) return rc;
+  if ((rc = check_subspace(S, who))) return rc;
+  UpdateArgs a{};
+  if ((rc = fill_update_members(a, n_members, noise_id, sign, fitness, n_noise, seeds, coef, who))) return rc;
+  a.w = p->w;
+  a.master = p->master;
+  a.n_alloc = p->n_alloc;
+  if (S->kind == COPES_SUBSPACE_TILES) {
+    a.tiles = S->tiles;
+    a.n_tiles = S->n_tiles;
+  } else {
+    a.index = S->index;
+    a.n_index = S->n_index;
+  }
+  a.fuse_commit = fuse_commit ? 1 : 0;
   if (S->kind == COPES_SUBSPACE_HASH_REPLAY)
     return launch_status(copes::launch_replay_update(p->dtype, a, replay_args(S), stream), who);
   return launch_status(copes::launch_update(S->kind, p->dtype, a, stream, 0), who);
+}
+
+// ---------------------------------------------------------------------- backup mode
+int copes_backup_save(const copes_backup_params *p, const copes_subspace *S, cudaStream_t stream) {
+  return run_backup_elementwise(copes::kBackupSave, p, S, 0, 0.0f, stream, "copes_backup_save");
+}
+
+int copes_backup_perturb(const copes_backup_params *p, const copes_subspace *S, uint64_t seed,
+                         float signed_sigma, cudaStream_t stream) {
+  if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "copes_backup_perturb: sigma is not finite");
+  return run_backup_elementwise(copes::kBackupPerturb, p, S, seed, signed_sigma, stream, "copes_backup_perturb");
+}
+
+int copes_backup_restore(const copes_backup_params *p, const copes_subspace *S, cudaStream_t stream) {
+  return run_backup_elementwise(copes::kBackupRestore, p, S, 0, 0.0f, stream, "copes_backup_restore");
+}
+
+int copes_backup_update(const copes_backup_params *p, const copes_subspace *S, int n_members,
+                        const int32_t *noise_id, const int8_t *sign, const float *fitness, int n_noise,
+                        const uint64_t *seeds, float coef, cudaStream_t stream) {
+  const char *who = "copes_backup_update";
+  UpdateArgs a{};
+  int rc = fill_update_members(a, n_members, noise_id, sign, fitness, n_noise, seeds, coef, who);
+  if (rc) return rc;
+  uint16_t *dev = nullptr;
+  if ((rc = check_backup(p, S, who, &dev))) return rc;
+  a.w = p->w;
+  a.n_alloc = p->n_alloc;
+  a.tiles = S->tiles;
+  a.n_tiles = S->n_tiles;
+  return launch_status(copes::launch_backup_update(a, dev, stream), who);
 }
 
 // ----------------------------------------------------------------------------- debug

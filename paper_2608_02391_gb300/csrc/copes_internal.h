@@ -185,6 +185,11 @@ cudaError_t launch_replay_elementwise(int op, int dtype, const ElemArgs &a, cons
 cudaError_t launch_replay_update(int dtype, const UpdateArgs &a, const ReplayArgs &r,
                                  cudaStream_t s);
 
+// CPU weight backup mode: `backup` is the device-accessible pointer of pinned host memory.
+enum BackupOp { kBackupSave = 0, kBackupPerturb = 1, kBackupRestore = 2 };
+cudaError_t launch_backup_elementwise(int op, const ElemArgs &a, uint16_t *backup, cudaStream_t s);
+cudaError_t launch_backup_update(const UpdateArgs &a, uint16_t *backup, cudaStream_t s);
+
 // Sets the calling thread's message reported by copes_last_error.
 void set_last_error(const char *message);
 
@@ -192,5 +197,6 @@ void set_last_error(const char *message);
 unsigned read_and_clear_es_errors();
 unsigned read_and_clear_partition_errors();
 unsigned read_and_clear_replay_errors();
+unsigned read_and_clear_backup_errors();
 
 }  // namespace copes

@@ -8,6 +8,9 @@ sync_step          one CoPES training step (Algorithm 1): every subspace's N_k =
                    members are evaluated under the same pre-update context, rewards are
                    standardised jointly (Eq. 12) or per subspace (Sec. 4.4 ablation), and
                    all K subspace updates are composed (Eq. 13) before the commit.
+backup_visit       round_robin_visit in the CPU weight backup mode (Supp. A.8): the
+                   context is saved to pinned host memory, members are perturbed from
+                   it, and restore copies it back; no fp32 master.
 population_visit   round_robin_visit with the population split across the ranks of a
                    process group, each rank holding a full replica of theta: a rank
                    evaluates its slice of the members, the N reward scalars are
@@ -63,6 +66,31 @@ def round_robin_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, ite
     _timed(events, "shape", lambda: copes.shape_fitness(rewards, cfg.shaping, out=f))
     coef = copes.step_coef(cfg.alpha, cfg.n_members, s_k, cfg.convention)
     _timed(events, "update", lambda: copes.update(arena, sub, nid, sign, f, seeds, coef, fuse_commit=True))
+    return f
+
+
+def backup_visit(arena: copes.BackupArena, sub: copes.SubspaceHandle, k: int, iteration: int,
+                 cfg: ESConfig, d: int, rewards: torch.Tensor,
+                 evaluate: Optional[Callable[[int], None]] = None,
+                 fitness_out: Optional[torch.Tensor] = None,
+                 events: Optional[dict] = None) -> torch.Tensor:
+    """One ES iteration on subspace k in the CPU weight backup mode: save the context of S
+    to the host backup, evaluate the N members perturbed from it, restore, shape, and
+    apply the update, which writes the new context to the weights and the backup."""
+    nid, sign, P = copes.member_table(cfg.n_members, cfg.pairing)
+    seeds = copes.member_seeds(cfg.base_seed, iteration, k, P)
+    s_k = sigma_k(cfg, d, sub.numel)
+    _timed(events, "save", lambda: copes.backup_save(arena, sub))
+    for i in range(cfg.n_members):
+        _timed(events, "perturb",
+               lambda: copes.backup_perturb(arena, sub, int(seeds[nid[i]]), float(sign[i]) * s_k))
+        if evaluate is not None:
+            evaluate(i)
+    _timed(events, "restore", lambda: copes.backup_restore(arena, sub))
+    f = fitness_out if fitness_out is not None else torch.empty_like(rewards)
+    _timed(events, "shape", lambda: copes.shape_fitness(rewards, cfg.shaping, out=f))
+    coef = copes.step_coef(cfg.alpha, cfg.n_members, s_k, cfg.convention)
+    _timed(events, "update", lambda: copes.backup_update(arena, sub, nid, sign, f, seeds, coef))
     return f
 
 

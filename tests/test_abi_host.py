@@ -179,3 +179,34 @@ def test_hash_replay_arguments_are_rejected_before_any_copy(lib):
     S = replay(K=65)
     assert lib.copes_update(ctypes.byref(p), ctypes.byref(S), 2, nid.ctypes.data_as(P), sg.ctypes.data_as(P),
                             fake, 1, seeds.ctypes.data_as(P), 0.1, 1, None) == copes.ERR_INVALID_ARG
+
+
+def test_backup_mode_arguments_are_rejected_before_any_launch(lib):
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    P = ctypes.c_void_p
+    tiles = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
+    idx = copes.Subspace(copes.SUBSPACE_INDICES, None, 0, fake, 4)
+    cases = [(None, tiles, copes.ERR_INVALID_ARG),
+             (copes.BackupParams(fake, None, 100), tiles, copes.ERR_INVALID_ARG),
+             (copes.BackupParams(fake + 2, fake, 100), tiles, copes.ERR_ALIGNMENT),
+             (copes.BackupParams(fake, fake + 8, 100), tiles, copes.ERR_ALIGNMENT),
+             (copes.BackupParams(fake, fake, 0), tiles, copes.ERR_SIZE),
+             (copes.BackupParams(fake, fake, 100), idx, copes.ERR_UNSUPPORTED)]
+    for prm, S, code in cases:
+        pp = None if prm is None else ctypes.byref(prm)
+        assert lib.copes_backup_save(pp, ctypes.byref(S), None) == code
+        assert lib.copes_backup_restore(pp, ctypes.byref(S), None) == code
+        assert lib.copes_backup_perturb(pp, ctypes.byref(S), 1, 1e-3, None) == code
+    prm = copes.BackupParams(fake, fake, 100)
+    assert lib.copes_backup_perturb(ctypes.byref(prm), ctypes.byref(tiles), 1, float("inf"), None) == \
+        copes.ERR_INVALID_ARG
+    nid = np.array([0, 0], np.int32)
+    sg = np.array([1, -1], np.int8)
+    seeds = np.zeros(1, np.uint64)
+    assert lib.copes_backup_update(ctypes.byref(prm), ctypes.byref(tiles), 300, nid.ctypes.data_as(P),
+                                   sg.ctypes.data_as(P), fake, 1, seeds.ctypes.data_as(P), 0.1, None) == \
+        copes.ERR_SIZE
+    assert lib.copes_backup_update(ctypes.byref(prm), ctypes.byref(idx), 2, nid.ctypes.data_as(P),
+                                   sg.ctypes.data_as(P), fake, 1, seeds.ctypes.data_as(P), 0.1, None) == \
+        copes.ERR_UNSUPPORTED
