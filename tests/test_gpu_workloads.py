@@ -210,6 +210,45 @@ def test_8b_type_groups_sampled(copes):
     copes.check()
 
 
+def test_8b_full_cc_loop_sampled(copes):
+    """The 8B workload as configured: 10 cooperative-coevolution cycles over the 4 type
+    groups (40 visits, N = 128 antithetic), through the round-robin schedule.  After every
+    visit the oracle recomputes the shaped fitness and the updated master at sampled
+    members of that subspace from the values they held before it, and the commit is checked
+    against the new master."""
+    from paper_2608_02391_gb300 import es
+    w = wl.workload("8b")
+    assert w.cycles == 10
+    arena, layout = make_arena(copes, w)
+    rng = np.random.default_rng(10)
+    subs, samples = [], []
+    for k in range(w.K):
+        sub = copes.subspace_build(layout, copes.PART_TENSOR_GROUPS, w.K, k, group_of=w.group_of,
+                                   tile_size=copes.DEFAULT_TILE)
+        subs.append(sub)
+        samples.append(sample_from_ranges(tile_ranges(sub), 1024, rng))
+    cfg = es.ESConfig(n_members=w.n_members, sigma=w.sigma, alpha=w.alpha, shaping=w.shaping)
+    rewards = wl.reward_stream(w, w.cycles * w.K)
+    nid, sign, P = copes.member_table(w.n_members, copes.ANTITHETIC)
+    sigma = np.float32(w.sigma)
+    coef = np.float32(copes.step_coef(w.alpha, w.n_members, float(sigma), copes.COEF_OPENAI))
+    for cycle in range(w.cycles):
+        for k in range(w.K):
+            idx = torch.from_numpy(samples[k]).cuda()
+            before = arena.master[idx].cpu().numpy()
+            r = rewards[cycle * w.K + k]
+            f = es.round_robin_visit(arena, subs[k], k, cycle, cfg, w.d, torch.from_numpy(r).cuda())
+            f_ref = oracle.shape_fitness(r, SHAPE[w.shaping])
+            assert_fitness_close(f.cpu().numpy(), f_ref)
+            seeds = copes.member_seeds(w.base_seed, cycle, k, P)
+            wj = oracle.noise_weights(nid, sign, f_ref, P)
+            _, exact, scale = oracle.update_at(samples[k].astype(np.uint64), before, seeds, wj, coef)
+            got = arena.master[idx].cpu().numpy()
+            assert_update_close(got, exact, scale)
+            assert np.array_equal(bf16_bits_of(arena.w, samples[k]), oracle.bf16_bits_array(got))
+    copes.check()
+
+
 # ---------------------------------------------------------------------------- 4B hash
 def test_4b_hash_partition_and_gather_visit(copes):
     w = wl.workload("4b-hash")
