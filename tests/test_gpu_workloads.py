@@ -328,6 +328,31 @@ def test_4b_hash_replay_visit_equals_list_path(copes):
     copes.check()
 
 
+def test_4b_hash_full_sweep_replay_sampled(copes):
+    """The 4B-hash workload as configured: one perturb / restore / update sweep over all 16
+    hash subspaces (N = 64), on replay subspaces (no index lists), each visit checked at
+    sampled members against the oracle; the members are found with the oracle's hash."""
+    w = wl.workload("4b-hash")
+    arena, _ = make_arena(copes, w)
+    tids = list(range(len(w.tensors)))
+    layout = copes.Layout(w.numel, tids)
+    subs = copes.hash_replay_partition(layout, w.K, w.partition_seed)
+    assert sum(s.numel for s in subs) == w.d
+    rng = np.random.default_rng(16)
+    off = oracle.layout(w.numel)
+    per_k = [[] for _ in range(w.K)]
+    sizes = np.array(w.numel, dtype=np.float64)
+    for t in rng.choice(len(w.tensors), size=24_000, p=sizes / sizes.sum()):
+        e = int(rng.integers(0, w.numel[t]))
+        per_k[oracle.hash_subspace(w.partition_seed, tids[t], e, w.K)].append(int(off[t]) + e)
+    rewards = wl.reward_stream(w, w.K)
+    for k in range(w.K):
+        sample = np.unique(np.array(per_k[k], dtype=np.int64))
+        assert sample.size > 1000
+        check_visit(copes, arena, subs[k], sample, w, k, 0, rewards[k])
+    copes.check()
+
+
 # ----------------------------------------------------------- beyond 2^34 global indices
 def test_counters_beyond_2_34(copes):
     """Tiles past global index 2^34 take the kernels' general counter path; a range
