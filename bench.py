@@ -320,11 +320,13 @@ def main():
     torch.cuda.synchronize()
     t0 = time.perf_counter()
     s0 = args.warmup + args.steps
+    e2e_events = {}  # the same per-kernel event records as the timed region
     for s in range(s0, s0 + args.e2e_steps):
         for k in range(wl.K):
             rebuild(k)
             r_dev.copy_(pinned[s * wl.K + k], non_blocking=True)
-            es.round_robin_visit(arena, subs[k], k, s, cfg, d, r_dev, fitness_out=f_all[k])
+            es.round_robin_visit(arena, subs[k], k, s, cfg, d, r_dev, fitness_out=f_all[k],
+                                 events=e2e_events)
         fit_host.copy_(f_all, non_blocking=True)
         torch.cuda.synchronize()
     e2e_s = max_over_ranks(time.perf_counter() - t0, "cuda")
