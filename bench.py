@@ -14,6 +14,11 @@ update per step, so value = parameters per step x steps / time.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl copes|reference]
 
+`--case 4b-sync` times the paper's Algorithm 1 step on the 4B set: a random equal-size
+chunk partition (K = 4, chunks of 65,536) resampled every step, N = 32 antithetic members
+split N_k = 8 per subspace, dimension-aware sigma_k, joint z-score and the composed
+update with coefficient alpha / N_k.
+
 `--case 4b-backup` times the 4B step in the CPU weight backup mode: bf16 weights on the
 GPU, the context in pinned host memory, no fp32 master.
 
@@ -63,11 +68,12 @@ def parse():
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice", "4b-backup"],
+    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice", "4b-backup", "4b-sync"],
                     help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling; "
                          "4b-hash: one sweep over the 16 hash subspaces of the 4B set (N=64); "
                          "4b-hash-slice: the same on 268M parameters, for profiling; "
-                         "4b-backup: the 4B step in the CPU weight backup mode (no fp32 master)")
+                         "4b-backup: the 4B step in the CPU weight backup mode (no fp32 master); "
+                         "4b-sync: Algorithm 1 on the 4B set (K=4 random chunks resampled each step)")
     ap.add_argument("--hash-mode", default="replay", choices=["replay", "lists"],
                     help="4b-hash: subspaces replayed from the partition seed, or int64 index lists")
     return ap.parse_args()
@@ -245,7 +251,7 @@ def make_arena(copes, torch, wl, layout):
 def main():
     args = parse()
     from paper_2608_02391_gb300 import workloads
-    wl = workloads.workload("4b" if args.case == "4b-backup" else args.case)
+    wl = workloads.workload("4b" if args.case in ("4b-backup", "4b-sync") else args.case)
     if args.impl == "reference":
         return run_reference(args, wl)
 
@@ -261,6 +267,8 @@ def main():
         return run_hash(args, wl, copes, es, torch, rank, world, local)
     if args.case == "4b-backup":
         return run_backup(args, wl, copes, es, torch, rank, world, local)
+    if args.case == "4b-sync":
+        return run_sync(args, wl, copes, es, torch, rank, world, local)
 
     layout = copes.Layout(wl.numel)
     d = wl.d
@@ -578,6 +586,95 @@ def run_backup(args, wl, copes, es, torch, rank, world, local):
         "clocks": clocks.summary(),
         "e2e": None,
         "gpu_launches": sum(counts.values()),
+    }
+    print(json.dumps(out), flush=True)
+
+
+def run_sync(args, wl, copes, es, torch, rank, world, local):
+    """Algorithm 1 on the 4B set: per step, a fresh random-chunk partition (K = 4), the
+    N_k = 8 members of every subspace perturbed under the same context, joint shaping and
+    the K composed updates + commit."""
+    from paper_2608_02391_gb300 import workloads
+    K, chunk = 4, 65536
+    layout = copes.Layout(wl.numel)
+    d = wl.d
+    arena = make_arena(copes, torch, wl, layout)
+    cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping="zscore",
+                      convention=copes.COEF_PAPER, dimension_aware=True)
+    total = args.warmup + args.steps
+    rewards = torch.from_numpy(workloads.reward_stream(wl, total)).cuda()
+
+    def step(s, events=None):
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record()
+        subs = es.build_subspaces(layout, "random_chunks", K, seed=1000 + s, chunk=chunk, tile_size=args.tile)
+        t1.record()
+        if events is not None:
+            events.setdefault("partition", []).append((t0, t1))
+        es.sync_step(arena, subs, s, cfg, d, rewards[s], joint=True, events=events)
+        return subs
+
+    for s in range(args.warmup):
+        step(s)
+    torch.cuda.synchronize()
+    copes.check()
+    events = {}
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        torch.cuda.synchronize()
+        start.record()
+        for s in range(args.warmup, args.warmup + args.steps):
+            subs = step(s, events)
+        end.record()
+        torch.cuda.synchronize()
+    ms = max_over_ranks(start.elapsed_time(end), "cuda")
+    copes.check()
+    if rank != 0:
+        return
+    per = {name: float(np.mean([a.elapsed_time(b) for a, b in lst])) for name, lst in events.items()}
+    counts = {name: len(lst) for name, lst in events.items()}
+    mean_dk = float(np.mean([s.numel for s in subs]))
+    peaks, _ = measured_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    clk = clocks.summary()
+    sm_mhz = clk["sm_mhz"] or 2070.0
+    props = torch.cuda.get_device_properties(local)
+    alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12
+    P = (wl.n_members // K) // 2
+    upd_tops = 28.0 * P * mean_dk / (per["update"] * 1e-3) / 1e12
+    upd_gbs = 10.0 * mean_dk / (per["update"] * 1e-3) / 1e9
+    # the update's roofline is the slower of its ALU and HBM bounds
+    t_alu = 28.0 * P * mean_dk / (alu_peak * 1e12)
+    t_hbm = 10.0 * mean_dk / (hbm * 1e9)
+    perturb_gbs = 6.0 * mean_dk / (per["perturb"] * 1e-3) / 1e9
+    value = job_throughput(world, d, args.steps, ms * 1e-3)
+    out = {
+        "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": "4B decoder-shaped bf16 set, fp32 master, Algorithm 1: K=4 random chunks "
+                               "(65,536) resampled per step, N=32 antithetic (N_k=8), dimension-aware sigma_k, "
+                               "joint z-score, coefficient alpha/N_k",
+                   "params": d, "K": K, "N": wl.n_members, "chunk": chunk, "sigma": wl.sigma, "alpha": wl.alpha,
+                   "tile": args.tile, "l2": "inputs larger than L2, no flush"},
+        "roofline": {"bound": "hbm", "kernel": "perturb", "achieved": perturb_gbs, "peak": hbm, "unit": "GB/s",
+                     "frac": perturb_gbs / hbm, "traffic": None, "peak_source": "measured"},
+        "kernels": {
+            "partition": {"ms": per["partition"], "launches": counts["partition"]},
+            "perturb": {"ms": per["perturb"], "launches": counts["perturb"], "GB/s": perturb_gbs,
+                        "frac_hbm": perturb_gbs / hbm},
+            "restore": {"ms": per["restore"], "launches": counts["restore"],
+                        "GB/s": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9},
+            "update_fused_commit": {"ms": per["update"], "launches": counts["update"], "Tops": upd_tops,
+                                    "GB/s": upd_gbs, "normals_per_elem": P,
+                                    "frac_of_slower_bound": max(t_alu, t_hbm) / (per["update"] * 1e-3),
+                                    "bound": "alu" if t_alu >= t_hbm else "hbm"},
+            "shape": {"ms": per["shape"], "launches": counts["shape"]},
+        },
+        "clocks": clk,
+        "e2e": None,
+        "gpu_launches": sum(v for k, v in counts.items() if k != "partition"),
     }
     print(json.dumps(out), flush=True)
 

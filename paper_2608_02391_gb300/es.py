@@ -97,7 +97,7 @@ def backup_visit(arena: copes.BackupArena, sub: copes.SubspaceHandle, k: int, it
 def sync_step(arena: copes.Arena, subs: Sequence[copes.SubspaceHandle], iteration: int,
               cfg: ESConfig, d: int, rewards: torch.Tensor,
               evaluate: Optional[Callable[[int, int], None]] = None,
-              joint: bool = True) -> torch.Tensor:
+              joint: bool = True, events: Optional[dict] = None) -> torch.Tensor:
     """Algorithm 1: N = cfg.n_members split into N_k = N / K per subspace; rewards is the
     device fp32 [N] vector laid out subspace by subspace (member i of subspace k at
     k N_k + i).  evaluate(k, i) runs while that member's perturbation is live."""
@@ -110,19 +110,23 @@ def sync_step(arena: copes.Arena, subs: Sequence[copes.SubspaceHandle], iteratio
     for k, sub in enumerate(subs):
         s_k = sigma_k(cfg, d, sub.numel)
         for i in range(n_k):
-            copes.perturb(arena, sub, int(seeds[k][nid[i]]), float(sign[i]) * s_k)
+            _timed(events, "perturb",
+                   lambda: copes.perturb(arena, sub, int(seeds[k][nid[i]]), float(sign[i]) * s_k))
             if evaluate is not None:
                 evaluate(k, i)
-        copes.restore(arena, sub)  # the next subspace is evaluated under the same context
+        # the next subspace is evaluated under the same context
+        _timed(events, "restore", lambda: copes.restore(arena, sub))
     if joint:
-        f = copes.shape_fitness(rewards, copes.SHAPE_ZSCORE if cfg.shaping == "zscore" else cfg.shaping)
+        f = _timed(events, "shape", lambda: copes.shape_fitness(
+            rewards, copes.SHAPE_ZSCORE if cfg.shaping == "zscore" else cfg.shaping))
     else:
         group = torch.arange(cfg.n_members, device=rewards.device, dtype=torch.int32) // n_k
-        f = copes.shape_fitness(rewards, copes.SHAPE_ZSCORE_GROUPED, group=group)
+        f = _timed(events, "shape", lambda: copes.shape_fitness(rewards, copes.SHAPE_ZSCORE_GROUPED, group=group))
     for k, sub in enumerate(subs):  # every g_k from the same pre-update theta (disjoint supports)
         s_k = sigma_k(cfg, d, sub.numel)
         coef = copes.step_coef(cfg.alpha, n_k, s_k, cfg.convention)
-        copes.update(arena, sub, nid, sign, f[k * n_k:(k + 1) * n_k], seeds[k], coef, fuse_commit=True)
+        _timed(events, "update", lambda: copes.update(arena, sub, nid, sign, f[k * n_k:(k + 1) * n_k], seeds[k],
+                                                      coef, fuse_commit=True))
     return f
 
 
