@@ -138,9 +138,12 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
   }
 }
 
-// One block per tile [tiles[2t], tiles[2t+1]).
+// One block per tile [tiles[2t], tiles[2t+1]).  3 resident blocks per SM leave 85 registers a
+// thread for G = 8 groups in flight (measured 2% faster than G = 4 at 4 blocks, the next best).
+constexpr int kElemBlocksPerSM = 3;
+
 template <int OP, typename WT, int G>
-__global__ void __launch_bounds__(kThreads) elem_tiles_kernel(const ElemArgs a) {
+__global__ void __launch_bounds__(kThreads, kElemBlocksPerSM) elem_tiles_kernel(const ElemArgs a) {
   const uint64_t t = blockIdx.x;
   const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
   if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
@@ -206,7 +209,7 @@ template <int OP, typename WT>
 static cudaError_t launch_elem_typed(int kind, const ElemArgs &a, cudaStream_t s) {
   if (kind == COPES_SUBSPACE_TILES) {
     if (a.n_tiles == 0) return cudaSuccess;
-    constexpr int G = 4;
+    constexpr int G = 8;
     elem_tiles_kernel<OP, WT, G><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
   } else {
     if (a.n_index == 0) return cudaSuccess;
