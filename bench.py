@@ -25,7 +25,8 @@ GPU, the context in pinned host memory, no fp32 master.
 `--case 4b-hash` times the non-contiguous workload instead: the same 4B set split by a
 per-element hash into K = 16 subspaces, N = 64 antithetic members, one step = one sweep
 over the 16 subspaces, with the subspaces replayed from the partition seed (default) or
-read from int64 index lists (`--hash-mode lists`).
+read from int64 index lists (`--hash-mode lists`), or read from index lists with each
+subspace's theta kept in list order (`--hash-mode gathered`).
 
 Prints one JSON line (rank 0).  Under torchrun each rank runs an independent replica on
 its own GPU (the path needs no exchange at this scope), timed with a barrier and the max
@@ -74,8 +75,9 @@ def parse():
                          "4b-hash-slice: the same on 268M parameters, for profiling; "
                          "4b-backup: the 4B step in the CPU weight backup mode (no fp32 master); "
                          "4b-sync: Algorithm 1 on the 4B set (K=4 random chunks resampled each step)")
-    ap.add_argument("--hash-mode", default="replay", choices=["replay", "lists"],
-                    help="4b-hash: subspaces replayed from the partition seed, or int64 index lists")
+    ap.add_argument("--hash-mode", default="replay", choices=["replay", "lists", "gathered"],
+                    help="4b-hash: subspaces replayed from the partition seed, int64 index lists, or "
+                         "index lists with a gathered (list-order) master per subspace")
     return ap.parse_args()
 
 
@@ -417,6 +419,9 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
         subs = copes.hash_replay_partition(layout, wl.K, wl.partition_seed)
     else:
         subs = copes.hash_partition(layout, wl.K, wl.partition_seed)
+        if args.hash_mode == "gathered":  # each subspace's theta in list order (contiguous reads)
+            for sub in subs:
+                copes.gather_master(arena, sub)
     cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping=wl.shaping)
     total_steps = args.warmup + args.steps
     rewards = torch.from_numpy(workloads.reward_stream(wl, total_steps * wl.K)).cuda()

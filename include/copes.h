@@ -108,6 +108,8 @@ typedef struct {
   int K;                   /* HASH_REPLAY: subspaces of the partition, 1 <= K <= COPES_MAX_K */
   int k;                   /* HASH_REPLAY: this subspace, 0 <= k < K                      */
   uint64_t seed;           /* HASH_REPLAY: the partition seed                             */
+  float *gathered;         /* INDICES, optional: device fp32 [n_index], the subspace's master
+                              values in list order (see copes_gather_master); NULL: none */
 } copes_subspace;
 
 /* Parameter layout: the model's tensors in order. */
@@ -248,6 +250,18 @@ int copes_hash_fill(const copes_layout_desc *layout, int K, uint64_t seed, void 
 int copes_hash_partition_static(const copes_layout_desc *layout, int K, uint64_t seed,
                                 int64_t *const *lists, const uint64_t *capacity,
                                 uint64_t *counts, cudaStream_t stream);
+
+/* Gathered master of an INDICES subspace (no counterpart in the paper: a memory-layout
+ * option for scattered subspaces).  With S->gathered set, perturb, restore, commit, init
+ * and update over S read theta from gathered[p] for the p-th index (and the update and
+ * init write it there) instead of master[index[p]]; master is not touched.  The results
+ * are those of the master path, bit for bit, while the master reads become contiguous
+ * (4 bytes per member instead of a 32-byte sector of master each).
+ *  copes_gather_master:  gathered[p] = master[index[p]]   (before the subspace's visits)
+ *  copes_scatter_master: master[index[p]] = gathered[p]   (to publish theta back)
+ * Both need S->kind == INDICES and S->gathered (16-byte aligned); asynchronous. */
+int copes_gather_master(const copes_params *p, const copes_subspace *S, cudaStream_t stream);
+int copes_scatter_master(const copes_params *p, const copes_subspace *S, cudaStream_t stream);
 
 /* HASH partition by replay (Supp. A.8 "Partition Replay": the partition is kept as its
  * seed and replayed, not stored as a parameter-level assignment).  Writes the layout's

@@ -50,7 +50,7 @@ class Subspace(ctypes.Structure):
                 ("index", ctypes.c_void_p), ("n_index", ctypes.c_uint64),
                 ("replay", ctypes.c_void_p), ("n_replay_tiles", ctypes.c_uint64),
                 ("n_replay_tensors", ctypes.c_int), ("K", ctypes.c_int), ("k", ctypes.c_int),
-                ("seed", ctypes.c_uint64)]
+                ("seed", ctypes.c_uint64), ("gathered", ctypes.c_void_p)]
 
 
 class BackupParams(ctypes.Structure):
@@ -96,6 +96,8 @@ SIGNATURES = {
     "copes_shape_fitness": (_I32, [_VP, _I32, _VP, _I32, _VP, _VP]),
     "copes_update": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _F32, _I32, _VP]),
     "copes_init_normal": (_I32, [_VP, _VP, _U64, _F32, _F32, _VP]),
+    "copes_gather_master": (_I32, [_VP, _VP, _VP]),
+    "copes_scatter_master": (_I32, [_VP, _VP, _VP]),
     "copes_backup_save": (_I32, [_VP, _VP, _VP]),
     "copes_backup_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
     "copes_backup_restore": (_I32, [_VP, _VP, _VP]),
@@ -224,6 +226,7 @@ class SubspaceHandle:
     tensor: torch.Tensor
     numel: int
     replay: Optional[Subspace] = None
+    gathered: Optional[torch.Tensor] = None  # INDICES: theta in list order (gather_master)
 
     def struct(self) -> Subspace:
         if self.kind == SUBSPACE_HASH_REPLAY:
@@ -231,8 +234,11 @@ class SubspaceHandle:
         if self.kind == SUBSPACE_TILES:
             return Subspace(SUBSPACE_TILES, self.tensor.data_ptr() if self.tensor.numel() else None,
                             self.tensor.shape[0], None, 0)
-        return Subspace(SUBSPACE_INDICES, None, 0,
-                        self.tensor.data_ptr() if self.tensor.numel() else None, self.tensor.numel())
+        S = Subspace(SUBSPACE_INDICES, None, 0, self.tensor.data_ptr() if self.tensor.numel() else None,
+                     self.tensor.numel())
+        if self.gathered is not None:
+            S.gathered = self.gathered.data_ptr()
+        return S
 
 
 def _tiles_result(count_fn, fill_fn, device, stream) -> SubspaceHandle:
@@ -350,6 +356,23 @@ def restore(arena: Arena, sub: SubspaceHandle, stream=None) -> None:
 def context_commit(arena: Arena, sub: SubspaceHandle, stream=None) -> None:
     S = sub.struct()
     _check(load().copes_context_commit(ctypes.byref(arena.params), ctypes.byref(S), _stream(stream)))
+
+
+def gather_master(arena: Arena, sub: SubspaceHandle, stream=None) -> torch.Tensor:
+    """Gives an INDICES subspace a gathered master (allocated here, n_index fp32) filled
+    with master[index[p]]; the ES steps over `sub` then read and update that copy."""
+    assert sub.kind == SUBSPACE_INDICES
+    if sub.gathered is None:
+        sub.gathered = torch.empty(max(sub.tensor.numel(), 1), dtype=torch.float32, device=sub.tensor.device)
+    S = sub.struct()
+    _check(load().copes_gather_master(ctypes.byref(arena.params), ctypes.byref(S), _stream(stream)))
+    return sub.gathered
+
+
+def scatter_master(arena: Arena, sub: SubspaceHandle, stream=None) -> None:
+    """Writes the gathered copy back: master[index[p]] = gathered[p]."""
+    S = sub.struct()
+    _check(load().copes_scatter_master(ctypes.byref(arena.params), ctypes.byref(S), _stream(stream)))
 
 
 def init_normal(arena: Arena, sub: SubspaceHandle, seed: int, mean: float, scale: float, stream=None) -> None:

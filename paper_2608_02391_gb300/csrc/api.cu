@@ -52,6 +52,9 @@ int check_params(const copes_params *p, const char *who) {
 
 int check_subspace(const copes_subspace *S, const char *who) {
   if (!S) return fail(COPES_ERR_INVALID_ARG, "%s: subspace is NULL", who);
+  if (S->gathered && S->kind != COPES_SUBSPACE_INDICES)
+    return fail(COPES_ERR_INVALID_ARG, "%s: a gathered master needs an INDICES subspace", who);
+  if (!aligned(S->gathered, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: gathered must be 16-byte aligned", who);
   if (S->kind == COPES_SUBSPACE_TILES) {
     if (S->n_tiles && !S->tiles) return fail(COPES_ERR_INVALID_ARG, "%s: tiles is NULL", who);
     if (!aligned(S->tiles, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: tiles must be 16-byte aligned", who);
@@ -139,6 +142,7 @@ ElemArgs elem_args(const copes_params *p, const copes_subspace *S) {
   } else {
     a.index = S->index;
     a.n_index = S->n_index;
+    a.gathered = S->kind == COPES_SUBSPACE_INDICES ? S->gathered : nullptr;
   }
   return a;
 }
@@ -514,6 +518,18 @@ int copes_context_commit(const copes_params *p, const copes_subspace *S, cudaStr
   return run_elementwise(copes::kOpRestore, p, S, 0, 0, 0.0f, 0.0f, stream, "copes_context_commit");
 }
 
+int copes_gather_master(const copes_params *p, const copes_subspace *S, cudaStream_t stream) {
+  if (S && (S->kind != COPES_SUBSPACE_INDICES || !S->gathered))
+    return fail(COPES_ERR_INVALID_ARG, "copes_gather_master: needs an INDICES subspace with gathered set");
+  return run_elementwise(copes::kOpGather, p, S, 0, 0, 0.0f, 0.0f, stream, "copes_gather_master");
+}
+
+int copes_scatter_master(const copes_params *p, const copes_subspace *S, cudaStream_t stream) {
+  if (S && (S->kind != COPES_SUBSPACE_INDICES || !S->gathered))
+    return fail(COPES_ERR_INVALID_ARG, "copes_scatter_master: needs an INDICES subspace with gathered set");
+  return run_elementwise(copes::kOpScatter, p, S, 0, 0, 0.0f, 0.0f, stream, "copes_scatter_master");
+}
+
 int copes_init_normal(const copes_params *p, const copes_subspace *S, uint64_t seed, float mean,
                       float scale, cudaStream_t stream) {
   return run_elementwise(copes::kOpInit, p, S, seed, COPES_TAG_INIT, scale, mean, stream,
@@ -629,6 +645,7 @@ int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
   } else {
     a.index = S->index;
     a.n_index = S->n_index;
+    a.gathered = S->kind == COPES_SUBSPACE_INDICES ? S->gathered : nullptr;
   }
   a.fuse_commit = fuse_commit ? 1 : 0;
   if (S->kind == COPES_SUBSPACE_HASH_REPLAY)

@@ -104,9 +104,11 @@ struct ElemArgs {
   float b;  // init: mean
   ScaledCoeffs coeffs;  // a * R's coefficients (perturb, init)
   uint32_t rk[20];      // Philox round keys of (seed_lo, seed_hi)
+  float *gathered;      // INDICES: theta in list order instead of master[index[p]] (or NULL)
 };
 
-enum ElemOp { kOpPerturb = 0, kOpRestore = 1, kOpInit = 2 };
+// kOpGather / kOpScatter copy theta between master and the gathered copy (INDICES only).
+enum ElemOp { kOpPerturb = 0, kOpRestore = 1, kOpInit = 2, kOpGather = 3, kOpScatter = 4 };
 
 struct UpdateArgs {
   void *w;
@@ -126,6 +128,7 @@ struct UpdateArgs {
   uint16_t noise_ptr[COPES_MAX_NOISE + 1];  // members of noise j: noise_member[ptr[j] .. ptr[j+1])
   uint16_t noise_member[COPES_MAX_MEMBERS];
   int8_t sign[COPES_MAX_MEMBERS];
+  float *gathered;  // INDICES: theta in list order instead of master[index[p]] (or NULL)
 };
 
 // ------------------------------------------------------------------------ launchers

@@ -161,7 +161,9 @@ __global__ void __launch_bounds__(kThreads, kElemBlocksPerSM) elem_tiles_kernel(
 // Gather form: the block's segment of the sorted index list is staged into shared memory
 // chunk by chunk (TMA bulk copies, double-buffered); each thread then handles its indices
 // of the chunk: load theta[g], one Philox word's normal, store w[g] (and theta[g] for init).
-template <int OP, typename WT>
+// GATH: theta lives in the subspace's gathered copy at the index's list position p
+// (a.gathered[p]) instead of master[g]; kOpGather / kOpScatter copy between the two.
+template <int OP, typename WT, bool GATH>
 __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) {
   __shared__ __align__(128) int64_t s_idx[2][kStageChunk];
   __shared__ __align__(8) uint64_t s_bar[2];
@@ -169,8 +171,9 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
   const uint64_t s0 = (uint64_t)blockIdx.x * kIndexSegment;
   const uint64_t s1 = min(s0 + (uint64_t)kIndexSegment, a.n_index);
   float *__restrict__ master = a.master;
+  float *__restrict__ gath = a.gathered;
   staged_index_segment(a.index, s0, s1, s_idx, s_bar, [] { flag_error(kErrStageTimeout); },
-                       [&](const int64_t *chunk, int cnt, uint64_t) {
+                       [&](const int64_t *chunk, int cnt, uint64_t first) {
     int64_t g[U];
     float th[U];
     bool ok[U];
@@ -183,38 +186,56 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
         flag_error(kErrIndexRange);
         ok[u] = false;
       }
-      th[u] = (OP != kOpInit && ok[u]) ? master[g[u]] : 0.0f;
+      const bool from_gathered = GATH && OP != kOpGather;
+      th[u] = (OP != kOpInit && ok[u]) ? (from_gathered ? gath[first + p] : master[g[u]]) : 0.0f;
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       if (!ok[u]) continue;
-      float v;
-      if (OP == kOpRestore) {
-        v = th[u];
+      if constexpr (OP == kOpGather) {
+        gath[first + threadIdx.x + kThreads * u] = th[u];
+        continue;
+      } else if constexpr (OP == kOpScatter) {
+        master[g[u]] = th[u];
+        continue;
       } else {
-        uint32_t x[4];
-        const uint64_t q = (uint64_t)g[u] >> 2;
-        philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, op_tag<OP>(), a.rk, x);
-        const uint32_t sel = (uint32_t)g[u] & 3u;
-        const uint32_t wd = sel == 0 ? x[0] : (sel == 1 ? x[1] : (sel == 2 ? x[2] : x[3]));
-        v = scaled_normal_plus(wd, a.coeffs, OP == kOpPerturb ? th[u] : a.b);
+        float v;
+        if (OP == kOpRestore) {
+          v = th[u];
+        } else {
+          uint32_t x[4];
+          const uint64_t q = (uint64_t)g[u] >> 2;
+          philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, op_tag<OP>(), a.rk, x);
+          const uint32_t sel = (uint32_t)g[u] & 3u;
+          const uint32_t wd = sel == 0 ? x[0] : (sel == 1 ? x[1] : (sel == 2 ? x[2] : x[3]));
+          v = scaled_normal_plus(wd, a.coeffs, OP == kOpPerturb ? th[u] : a.b);
+        }
+        if (OP == kOpInit) {
+          if (GATH) gath[first + threadIdx.x + kThreads * u] = v;
+          else master[g[u]] = v;
+        }
+        WStore<WT>::one(a.w, (uint64_t)g[u], v);
       }
-      if (OP == kOpInit) master[g[u]] = v;
-      WStore<WT>::one(a.w, (uint64_t)g[u], v);
     }
   });
 }
 
 template <int OP, typename WT>
 static cudaError_t launch_elem_typed(int kind, const ElemArgs &a, cudaStream_t s) {
-  if (kind == COPES_SUBSPACE_TILES) {
+  if constexpr (OP == kOpGather || OP == kOpScatter) {
+    if (kind != COPES_SUBSPACE_INDICES || !a.gathered) return cudaErrorInvalidValue;
+    if (a.n_index == 0) return cudaSuccess;
+    const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
+    elem_index_kernel<OP, WT, true><<<(unsigned)blocks, kThreads, 0, s>>>(a);
+  } else if (kind == COPES_SUBSPACE_TILES) {
     if (a.n_tiles == 0) return cudaSuccess;
     constexpr int G = 8;
     elem_tiles_kernel<OP, WT, G><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
   } else {
     if (a.n_index == 0) return cudaSuccess;
     const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
-    elem_index_kernel<OP, WT><<<(unsigned)blocks, kThreads, 0, s>>>(a);
+    if (a.gathered) elem_index_kernel<OP, WT, true><<<(unsigned)blocks, kThreads, 0, s>>>(a);
+    else elem_index_kernel<OP, WT, false><<<(unsigned)blocks, kThreads, 0, s>>>(a);
   }
   return cudaGetLastError();
 }
@@ -229,6 +250,8 @@ cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, c
   switch (op) {
     case kOpPerturb: return launch_elem_op<kOpPerturb>(kind, dtype, a, s);
     case kOpRestore: return launch_elem_op<kOpRestore>(kind, dtype, a, s);
+    case kOpGather: return launch_elem_op<kOpGather>(kind, dtype, a, s);
+    case kOpScatter: return launch_elem_op<kOpScatter>(kind, dtype, a, s);
     default: return launch_elem_op<kOpInit>(kind, dtype, a, s);
   }
 }
@@ -325,7 +348,8 @@ __global__ void __launch_bounds__(kThreads, kUpdateBlocksPerSM) update_tiles_ker
 
 // Gather form of the update: indices staged through shared memory as in
 // elem_index_kernel; every index regenerates the P normals from its own Philox word.
-template <typename WT, bool COMMIT>
+// GATH: theta is read from and written to the gathered copy at the list position.
+template <typename WT, bool COMMIT, bool GATH>
 __global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_constant__ UpdateArgs a) {
   __shared__ float s_w[COPES_MAX_NOISE];
   __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
@@ -336,9 +360,10 @@ __global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_con
   const uint64_t s0 = (uint64_t)blockIdx.x * kIndexSegment;
   const uint64_t s1 = min(s0 + (uint64_t)kIndexSegment, a.n_index);
   float *__restrict__ master = a.master;
+  float *__restrict__ gath = a.gathered;
   const int P = a.n_noise;
   staged_index_segment(a.index, s0, s1, s_idx, s_bar, [] { flag_error(kErrStageTimeout); },
-                       [&](const int64_t *chunk, int cnt, uint64_t) {
+                       [&](const int64_t *chunk, int cnt, uint64_t first) {
     for (int p0 = threadIdx.x; p0 < cnt; p0 += kThreads * U) {
       int64_t g[U];
       float acc[U];
@@ -375,8 +400,9 @@ __global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_con
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         if (!ok[u]) continue;
-        const float v = __fmaf_rn(a.coef, acc[u], master[g[u]]);
-        master[g[u]] = v;
+        float *th = GATH ? &gath[first + p0 + kThreads * u] : &master[g[u]];
+        const float v = __fmaf_rn(a.coef, acc[u], *th);
+        *th = v;
         if (COMMIT) WStore<WT>::one(a.w, (uint64_t)g[u], v);
       }
     }
@@ -391,7 +417,8 @@ static cudaError_t launch_update_typed(int kind, const UpdateArgs &a, cudaStream
   } else {
     if (a.n_index == 0) return cudaSuccess;
     const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
-    update_index_kernel<WT, COMMIT><<<(unsigned)blocks, kThreads, 0, s>>>(a);
+    if (a.gathered) update_index_kernel<WT, COMMIT, true><<<(unsigned)blocks, kThreads, 0, s>>>(a);
+    else update_index_kernel<WT, COMMIT, false><<<(unsigned)blocks, kThreads, 0, s>>>(a);
   }
   return cudaGetLastError();
 }

@@ -210,3 +210,18 @@ def test_backup_mode_arguments_are_rejected_before_any_launch(lib):
     assert lib.copes_backup_update(ctypes.byref(prm), ctypes.byref(idx), 2, nid.ctypes.data_as(P),
                                    sg.ctypes.data_as(P), fake, 1, seeds.ctypes.data_as(P), 0.1, None) == \
         copes.ERR_UNSUPPORTED
+
+
+def test_gathered_master_arguments_are_rejected_before_any_launch(lib):
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    p = copes.Params(fake, fake, 100, copes.BF16)
+    tiles = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
+    tiles.gathered = fake
+    assert lib.copes_perturb(ctypes.byref(p), ctypes.byref(tiles), 1, 1e-3, None) == copes.ERR_INVALID_ARG
+    idx = copes.Subspace(copes.SUBSPACE_INDICES, None, 0, fake, 4)
+    assert lib.copes_gather_master(ctypes.byref(p), ctypes.byref(idx), None) == copes.ERR_INVALID_ARG
+    assert lib.copes_scatter_master(ctypes.byref(p), ctypes.byref(idx), None) == copes.ERR_INVALID_ARG
+    idx.gathered = fake + 4
+    assert lib.copes_gather_master(ctypes.byref(p), ctypes.byref(idx), None) == copes.ERR_ALIGNMENT
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(idx), None) == copes.ERR_ALIGNMENT

@@ -236,3 +236,41 @@ def test_device_range_checks_report_without_faulting(copes):
         copes.check()
     assert e.value.code == copes.ERR_DEVICE_CHECK
     copes.check()  # cleared
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_gathered_master_equals_master_path(copes, dtype):
+    """An INDICES subspace with a gathered master: perturb, restore, update and init give
+    the master path's results bit for bit, master stays untouched until the scatter, and
+    the scatter publishes the gathered values."""
+    theta = theta_np(seed=21)
+    a1, a2 = make(copes, dtype, theta), make(copes, dtype, theta)
+    s1 = subspace(copes, "indices", RANGES, 0)
+    s2 = subspace(copes, "indices", RANGES, 0)
+    copes.gather_master(a2, s2)
+    inside = mask_of(RANGES)
+    assert np.array_equal(s2.gathered.cpu().numpy(), theta[inside])
+    for seed, ss in [(5, 1e-3), (6, -2e-3)]:
+        copes.perturb(a1, s1, seed, ss)
+        copes.perturb(a2, s2, seed, ss)
+        assert np.array_equal(w_bits(a1), w_bits(a2))
+    copes.restore(a1, s1)
+    copes.restore(a2, s2)
+    assert np.array_equal(w_bits(a1), w_bits(a2))
+    nid, sign, P = copes.member_table(32, copes.ANTITHETIC)
+    f = torch.linspace(-1, 1, 32, device="cuda")
+    seeds = copes.member_seeds(33, 0, 1, P)
+    copes.update(a1, s1, nid, sign, f, seeds, 0.3)
+    copes.update(a2, s2, nid, sign, f, seeds, 0.3)
+    assert np.array_equal(w_bits(a1), w_bits(a2))
+    assert np.array_equal(a2.master.cpu().numpy(), theta)  # untouched until the scatter
+    m1 = a1.master.cpu().numpy()
+    assert np.array_equal(s2.gathered.cpu().numpy().view(np.uint32), m1[inside].view(np.uint32))
+    copes.scatter_master(a2, s2)
+    assert np.array_equal(a2.master.cpu().numpy().view(np.uint32), m1.view(np.uint32))
+    copes.init_normal(a1, s1, 9, 0.0, 0.02)
+    copes.init_normal(a2, s2, 9, 0.0, 0.02)
+    assert np.array_equal(w_bits(a1), w_bits(a2))
+    assert np.array_equal(s2.gathered.cpu().numpy().view(np.uint32),
+                          a1.master.cpu().numpy()[inside].view(np.uint32))
+    copes.check()
