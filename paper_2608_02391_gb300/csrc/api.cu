@@ -229,8 +229,9 @@ int copes_check(cudaStream_t stream) {
   if ((e = cudaGetLastError()) != cudaSuccess) return cuda_fail(e, "copes_check");
   if (bits)
     return fail(COPES_ERR_DEVICE_CHECK,
-                "copes_check: a kernel skipped out-of-range accesses (bits 0x%x: 1 = tile outside "
-                "the arena, 2 = gather index outside the arena, 4 = partition workspace)",
+                "copes_check: a kernel's own check failed and it skipped the work (bits 0x%x: 1 = tile "
+                "outside the arena, 2 = gather index outside the arena, 4 = inconsistent partition "
+                "workspace or replay table, 8 = a bulk-copy wait ran out)",
                 bits);
   return COPES_OK;
 }
