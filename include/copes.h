@@ -213,9 +213,13 @@ int copes_tiles_from_ranges(const uint64_t *begin, const uint64_t *end, int n_ra
 /* RANDOM_CHUNKS map: chunk c (global indices [c chunk, (c+1) chunk)) gets key = word 0
  * of Philox(seed; c, 0, COPES_TAG_CHUNK); chunks ranked by (key, c) go to subspace
  * floor(rank K / n_chunks), so subspace sizes differ by at most one chunk.  Writes
- * n_chunks uint32 to the device array map.  n_chunks <= 2^20. */
+ * n_chunks uint32 to the device array map.  n_chunks <= 2^20.  workspace: device memory
+ * of copes_random_chunk_map_workspace_bytes(n_chunks) bytes (8 per chunk, the count
+ * rounded up to a power of two of at least 4,096), 16-byte aligned; the ranks come from
+ * a sort of the chunks' keys there.  Asynchronous. */
+size_t copes_random_chunk_map_workspace_bytes(uint64_t n_chunks);
 int copes_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,
-                           cudaStream_t stream);
+                           void *workspace, size_t workspace_bytes, cudaStream_t stream);
 
 /* HASH partition, phase 1: element e of tensor tid goes to subspace
  * floor(x K / 2^32) with x = word (e & 3) of Philox(seed; e >> 2, tid, COPES_TAG_PARTITION).

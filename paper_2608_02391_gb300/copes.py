@@ -83,7 +83,8 @@ SIGNATURES = {
     "copes_member_seed": (_U64, [_U64, _U32, _U32, _U32]),
     "copes_subspace_build": (_I32, [_VP, _VP, _I32, _U64, _VP, _VP, _U64, _VP, _VP]),
     "copes_tiles_from_ranges": (_I32, [_VP, _VP, _I32, _U64, _VP, _U64, _VP, _VP]),
-    "copes_random_chunk_map": (_I32, [_U64, _I32, _U64, _VP, _VP]),
+    "copes_random_chunk_map_workspace_bytes": (_SZ, [_U64]),
+    "copes_random_chunk_map": (_I32, [_U64, _I32, _U64, _VP, _VP, _SZ, _VP]),
     "copes_hash_workspace_bytes": (_SZ, [_VP, _I32]),
     "copes_hash_count": (_I32, [_VP, _I32, _U64, _VP, _SZ, _VP, _VP]),
     "copes_hash_fill": (_I32, [_VP, _I32, _U64, _VP, _SZ, _VP, _VP]),
@@ -278,8 +279,14 @@ def subspace_build(layout: Layout, mode: int, K: int, k: int, seed: int = 0, chu
 
 
 def random_chunk_map(n_chunks: int, K: int, seed: int, device="cuda", stream=None) -> torch.Tensor:
+    """copes_random_chunk_map with a torch-allocated sort workspace."""
+    L = load()
     out = torch.empty(n_chunks, dtype=torch.int32, device=device)
-    _check(load().copes_random_chunk_map(n_chunks, K, seed, _ptr(out), _stream(stream)))
+    nbytes = L.copes_random_chunk_map_workspace_bytes(n_chunks)
+    ws = torch.empty(max(nbytes, 16), dtype=torch.uint8, device=device)
+    _check(L.copes_random_chunk_map(n_chunks, K, seed, _ptr(out), _ptr(ws), nbytes, _stream(stream)))
+    if stream is not None:
+        ws.record_stream(stream)  # freed in stream order with the sort's kernels
     return out
 
 

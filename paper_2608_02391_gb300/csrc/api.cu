@@ -352,14 +352,24 @@ int copes_subspace_build(const copes_layout_desc *layout, const copes_partition_
   return emit_tiles(r, tile_size, tiles, capacity, count, stream, who);
 }
 
-int copes_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,
-                           cudaStream_t stream) {
+size_t copes_random_chunk_map_workspace_bytes(uint64_t n_chunks) {
+  if (n_chunks == 0 || n_chunks > (1ull << 20)) return 0;
+  return (size_t)copes::chunk_sort_size(n_chunks) * 8;
+}
+
+int copes_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map, void *workspace,
+                           size_t workspace_bytes, cudaStream_t stream) {
   const char *who = "copes_random_chunk_map";
   if (n_chunks == 0 || n_chunks > (1ull << 20))
     return fail(COPES_ERR_SIZE, "%s: n_chunks must be in [1, 2^20]", who);
   if (K < 1) return fail(COPES_ERR_INVALID_ARG, "%s: K must be >= 1", who);
   if (!map) return fail(COPES_ERR_INVALID_ARG, "%s: map is NULL", who);
-  return launch_status(copes::launch_random_chunk_map(n_chunks, K, seed, map, stream), who);
+  const size_t need = copes_random_chunk_map_workspace_bytes(n_chunks);
+  if (!workspace || workspace_bytes < need)
+    return fail(COPES_ERR_WORKSPACE, "%s: a workspace of %zu bytes is needed", who, need);
+  if (!aligned(workspace, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: workspace must be 16-byte aligned", who);
+  return launch_status(copes::launch_random_chunk_map(n_chunks, K, seed, map,
+                                                      static_cast<uint64_t *>(workspace), stream), who);
 }
 
 // ----------------------------------------------------------------------- hash partition

@@ -165,8 +165,10 @@ cudaError_t launch_hash_scan(const uint32_t *hist, uint64_t n_htiles, int K, uin
 cudaError_t launch_hash_scatter(const HashTensor *tensors, int n_tensors, uint64_t n_htiles,
                                 int K, uint64_t seed, const uint64_t *offsets,
                                 int64_t *const *lists, cudaStream_t s);
+// keys: workspace of chunk_sort_size(n_chunks) uint64.
+uint64_t chunk_sort_size(uint64_t n_chunks);
 cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,
-                                    cudaStream_t s);
+                                    uint64_t *keys, cudaStream_t s);
 
 // Partition replay: subspace k of the hash partition (K, seed), recomputed per hash tile
 // from the replay table: one HashTensor per non-empty tensor (layout order), then, from

@@ -139,42 +139,88 @@ __global__ void __launch_bounds__(kPartThreads) hash_scatter_kernel(
   }
 }
 
-// Random chunk map: chunk c has key = word 0 of Philox(seed; c, 0, CHUNK tag); its rank
-// under (key, c) order is counted against every other chunk; map[c] = rank K / n.
-__global__ void __launch_bounds__(kPartThreads) chunk_rank_kernel(uint64_t n, int K, uint64_t seed,
-                                                                  uint32_t *map) {
-  __shared__ uint32_t s_key[1024];
-  const uint64_t c = (uint64_t)blockIdx.x * kPartThreads + threadIdx.x;
-  const uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
-  uint32_t mine = 0;
-  if (c < n) {
+// Random chunk map: chunk c has key = word 0 of Philox(seed; c, 0, CHUNK tag) and goes to
+// subspace floor(rank K / n), rank = its position in (key, c) order.  The composite keys
+// (key << 20) | c (c < 2^20) are distinct, so the ranks are the positions after sorting
+// them: a bitonic sort over the caller's workspace (N = a power of two >= n, padded with
+// the largest key), with every 4,096-key tile sorted and merged in shared memory and
+// only the strides of 4,096 and more done by global-memory passes.
+constexpr uint64_t kSortTile = 4096;
+constexpr int kSortThreads = 512;
+
+__global__ void __launch_bounds__(kSortThreads) chunk_keys_kernel(uint64_t n, uint64_t N, uint64_t seed,
+                                                                   uint64_t *A) {
+  const uint64_t i = (uint64_t)blockIdx.x * kSortThreads + threadIdx.x;
+  if (i >= N) return;
+  if (i < n) {
     uint32_t x[4];
-    philox4x32_10((uint32_t)c, (uint32_t)(c >> 32), 0u, COPES_TAG_CHUNK, k0, k1, x);
-    mine = x[0];
+    philox4x32_10((uint32_t)i, (uint32_t)(i >> 32), 0u, COPES_TAG_CHUNK, (uint32_t)seed,
+                  (uint32_t)(seed >> 32), x);
+    A[i] = ((uint64_t)x[0] << 20) | i;
+  } else {
+    A[i] = ~0ull;
   }
-  uint64_t less = 0;
-  for (uint64_t base = 0; base < n; base += 1024) {
-    for (int i = threadIdx.x; i < 1024; i += kPartThreads) {
-      const uint64_t cc = base + i;
-      uint32_t key = 0xFFFFFFFFu;
-      if (cc < n) {
-        uint32_t x[4];
-        philox4x32_10((uint32_t)cc, (uint32_t)(cc >> 32), 0u, COPES_TAG_CHUNK, k0, k1, x);
-        key = x[0];
-      }
-      s_key[i] = key;
-    }
-    __syncthreads();
-    if (c < n) {
-      const int m = (int)min((uint64_t)1024, n - base);
-      for (int i = 0; i < m; ++i) {
-        const uint32_t key = s_key[i];
-        less += (key < mine) || (key == mine && base + i < c);
+}
+
+// One compare-exchange step (stage k, stride j) over a tile held in shared memory; the
+// direction of each pair comes from its global index.
+__device__ __forceinline__ void bitonic_smem_step(uint64_t *s, uint64_t base, uint64_t k, uint64_t j) {
+  for (uint32_t t = threadIdx.x; t < kSortTile; t += kSortThreads) {
+    const uint32_t l = t ^ (uint32_t)j;
+    if (l > t) {
+      const bool up = ((base + t) & k) == 0;
+      const uint64_t a = s[t], b = s[l];
+      if ((a > b) == up) {
+        s[t] = b;
+        s[l] = a;
       }
     }
-    __syncthreads();
   }
-  if (c < n) map[c] = (uint32_t)((less * (uint64_t)K) / n);
+  __syncthreads();
+}
+
+// k_stage == 0: sort every tile (stages 2 .. kSortTile).  Otherwise: the strides below
+// kSortTile of stage k_stage.
+__global__ void __launch_bounds__(kSortThreads) bitonic_tile_kernel(uint64_t *A, uint64_t k_stage) {
+  __shared__ uint64_t s[kSortTile];
+  const uint64_t base = (uint64_t)blockIdx.x * kSortTile;
+  for (uint32_t t = threadIdx.x; t < kSortTile; t += kSortThreads) s[t] = A[base + t];
+  __syncthreads();
+  if (k_stage == 0) {
+    for (uint64_t k = 2; k <= kSortTile; k <<= 1)
+      for (uint64_t j = k >> 1; j > 0; j >>= 1) bitonic_smem_step(s, base, k, j);
+  } else {
+    for (uint64_t j = kSortTile >> 1; j > 0; j >>= 1) bitonic_smem_step(s, base, k_stage, j);
+  }
+  for (uint32_t t = threadIdx.x; t < kSortTile; t += kSortThreads) A[base + t] = s[t];
+}
+
+__global__ void __launch_bounds__(kSortThreads) bitonic_global_kernel(uint64_t *A, uint64_t N, uint64_t j,
+                                                                      uint64_t k) {
+  const uint64_t i = (uint64_t)blockIdx.x * kSortThreads + threadIdx.x;
+  if (i >= N) return;
+  const uint64_t l = i ^ j;
+  if (l > i) {
+    const bool up = (i & k) == 0;
+    const uint64_t a = A[i], b = A[l];
+    if ((a > b) == up) {
+      A[i] = b;
+      A[l] = a;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kSortThreads) chunk_map_kernel(const uint64_t *A, uint64_t n, int K,
+                                                                 uint32_t *map) {
+  const uint64_t i = (uint64_t)blockIdx.x * kSortThreads + threadIdx.x;
+  if (i >= n) return;
+  map[A[i] & 0xFFFFFull] = (uint32_t)((i * (uint64_t)K) / n);
+}
+
+uint64_t chunk_sort_size(uint64_t n_chunks) {
+  uint64_t N = kSortTile;
+  while (N < n_chunks) N <<= 1;
+  return N;
 }
 
 cudaError_t launch_hash_hist(const HashTensor *tensors, int n_tensors, uint64_t n_htiles, int K,
@@ -205,9 +251,19 @@ cudaError_t launch_hash_scatter(const HashTensor *tensors, int n_tensors, uint64
 }
 
 cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,
-                                    cudaStream_t s) {
-  const unsigned blocks = (unsigned)((n_chunks + kPartThreads - 1) / kPartThreads);
-  chunk_rank_kernel<<<blocks, kPartThreads, 0, s>>>(n_chunks, K, seed, map);
+                                    uint64_t *keys, cudaStream_t s) {
+  const uint64_t N = chunk_sort_size(n_chunks);
+  const unsigned gblocks = (unsigned)((N + kSortThreads - 1) / kSortThreads);
+  const unsigned tiles = (unsigned)(N / kSortTile);
+  chunk_keys_kernel<<<gblocks, kSortThreads, 0, s>>>(n_chunks, N, seed, keys);
+  bitonic_tile_kernel<<<tiles, kSortThreads, 0, s>>>(keys, 0);
+  for (uint64_t k = 2 * kSortTile; k <= N; k <<= 1) {
+    for (uint64_t j = k >> 1; j >= kSortTile; j >>= 1)
+      bitonic_global_kernel<<<gblocks, kSortThreads, 0, s>>>(keys, N, j, k);
+    bitonic_tile_kernel<<<tiles, kSortThreads, 0, s>>>(keys, k);
+  }
+  const unsigned mblocks = (unsigned)((n_chunks + kSortThreads - 1) / kSortThreads);
+  chunk_map_kernel<<<mblocks, kSortThreads, 0, s>>>(keys, n_chunks, K, map);
   return cudaGetLastError();
 }
 

@@ -127,8 +127,16 @@ def test_invalid_arguments_are_rejected_before_any_launch(lib):
                                 None) == copes.ERR_WORKSPACE
     assert lib.copes_hash_count(ctypes.byref(L.desc), 65, 1, fake, need, counts.ctypes.data_as(P),
                                 None) == copes.ERR_INVALID_ARG
-    assert lib.copes_random_chunk_map(0, 4, 1, fake, None) == copes.ERR_SIZE
-    assert lib.copes_random_chunk_map((1 << 20) + 1, 4, 1, fake, None) == copes.ERR_SIZE
+    assert lib.copes_random_chunk_map(0, 4, 1, fake, fake, 1 << 20, None) == copes.ERR_SIZE
+    assert lib.copes_random_chunk_map((1 << 20) + 1, 4, 1, fake, fake, 1 << 24, None) == copes.ERR_SIZE
+    # the sort workspace: 8 bytes per chunk, the count rounded up to a power of two >= 4096
+    assert lib.copes_random_chunk_map_workspace_bytes(1) == 8 * 4096
+    assert lib.copes_random_chunk_map_workspace_bytes(4097) == 8 * 8192
+    assert lib.copes_random_chunk_map_workspace_bytes(1 << 20) == 8 << 20
+    assert lib.copes_random_chunk_map_workspace_bytes((1 << 20) + 1) == 0
+    assert lib.copes_random_chunk_map(5000, 4, 1, fake, fake, 8 * 4096, None) == copes.ERR_WORKSPACE
+    assert lib.copes_random_chunk_map(5000, 4, 1, fake, None, 8 * 8192, None) == copes.ERR_WORKSPACE
+    assert lib.copes_random_chunk_map(5000, 4, 1, fake, fake + 8, 8 * 8192, None) == copes.ERR_ALIGNMENT
     spec = copes.PartitionSpec(copes.PART_HASH, 4, 0, 0, None)
     cnt = ctypes.c_uint64()
     assert lib.copes_subspace_build(ctypes.byref(L.desc), ctypes.byref(spec), 0, 100, None, None, 0,

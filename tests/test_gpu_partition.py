@@ -52,7 +52,8 @@ def test_group_tiles(copes):
         check_tiles(sub, oracle.group_ranges(ODD_LAYOUT, groups, k), 512)
 
 
-@pytest.mark.parametrize("n_chunks,K", [(1, 1), (10, 4), (61, 8), (3000, 16), (70_000, 7)])
+@pytest.mark.parametrize("n_chunks,K", [(1, 1), (10, 4), (61, 8), (3000, 16), (4096, 3), (4097, 5),
+                                         (8192, 64), (70_000, 7), (1 << 20, 13)])
 def test_random_chunk_map(copes, n_chunks, K):
     seed = 1088 + n_chunks
     got = copes.random_chunk_map(n_chunks, K, seed).cpu().numpy().view(np.uint32)
