@@ -4,7 +4,7 @@
 // tiles; each warp streams through its 2,048-element stretch of every tile (replay_stream):
 //  - it hashes 32 four-element groups at a time -- one Philox4x32-10 call per group at
 //    counter (e >> 2, tensor id, TAG_PARTITION), bucket floor(x K / 2^32) per word -- and
-//    appends the tile offsets of the members of subspace k to its shared-memory buffer;
+//    appends the members of subspace k to its shared-memory buffer;
 //  - whenever the buffer holds a full batch, the warp processes it one member per lane,
 //    exactly as the gather kernels process an index list: perturb / restore / commit /
 //    init, or the fused update regenerating the P normals of each element.
@@ -64,11 +64,12 @@ __device__ __forceinline__ ReplayTile replay_tile(const ReplayArgs &r, uint64_t 
 
 // Warp-streamed replay over the block's hash tiles.  Each warp owns a 2,048-element
 // stretch of every tile and walks it 32 groups (one per lane) at a time: it hashes the
-// groups, appends the members of subspace r.k to its shared-memory buffer through a shuffle scan of the per-lane counts, and whenever
-// the buffer holds BATCH members it processes them, BATCH / 32 per lane, every lane
-// busy, so the hashing (ALU) interleaves with the members' scattered loads and stores.
-// The warps' leftovers (fewer than BATCH each) are pooled and processed by the whole
-// block at the end.  Every warp runs the same iterations, so full-warp shuffles are safe.
+// groups, appends the members of subspace r.k to its shared-memory buffer with one ballot
+// per word slot, and whenever the buffer holds BATCH members it processes them, BATCH / 32
+// per lane, every lane busy, so the hashing (ALU) interleaves with the members' scattered
+// loads and stores.  The warps' leftovers (fewer than BATCH each) are pooled and processed
+// by the whole block at the end; `flush` then runs once.  Every warp runs the same
+// iterations, so the full-warp ballots and shuffles see all 32 lanes.
 template <int BATCH, typename Fn, typename Flush>
 __device__ __forceinline__ void replay_stream(const ReplayArgs &r, uint64_t n_alloc, uint32_t *wbuf,
                                               uint64_t (*s_g0)[kReplayTilesPerBlock], uint32_t *pool,
