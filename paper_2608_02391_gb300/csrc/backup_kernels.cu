@@ -113,7 +113,7 @@ __global__ void __launch_bounds__(kThreads) backup_update_kernel(const __grid_co
         uint32_t x[4];
         philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, x);
         float eps[4];
-        normals4(x, eps);
+        normals4_x2(x, eps);
 #pragma unroll
         for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
       }

@@ -149,6 +149,49 @@ __device__ __forceinline__ void normals4(const uint32_t (&w)[4], float (&eps)[4]
   for (int e = 0; e < 4; ++e) eps[e] = __fmul_rn(x[e], r[e]);
 }
 
+// normals4 with the central polynomial on packed fp32 pairs, its coefficients (c, c)
+// compile-time constants: bit-identical to normals4, at fewer issue slots and without
+// coefficient registers.
+__device__ __forceinline__ void normals4_x2(const uint32_t (&w)[4], float (&eps)[4]) {
+  COPES_UNIT_COEFFS;
+  unsigned long long c2[COPES_NORMAL_CENTRAL_DEGREE + 1];
+#pragma unroll
+  for (int k = 0; k <= COPES_NORMAL_CENTRAL_DEGREE; ++k) {
+    const unsigned long long b = __float_as_uint(unit_central[k]);
+    c2[k] = (b << 32) | b;
+  }
+  float x[4], r[4];
+  normal_parts4_x2(w, c2, unit_tail, x, r);
+#pragma unroll
+  for (int e = 0; e < 4; ++e) eps[e] = __fmul_rn(x[e], r[e]);
+}
+
+// Two standard normals from two words (of different Philox blocks), their central
+// polynomials evaluated as one packed pair with compile-time coefficients and a single
+// warp vote for the tail: bit-identical to two normal_from_word calls.
+__device__ __forceinline__ void normal_pair_x2(uint32_t wa, uint32_t wb, float &ea, float &eb) {
+  COPES_UNIT_COEFFS;
+  const float xa = lattice_x(wa), xb = lattice_x(wb);
+  const float La = lg2_approx(__fmaf_rn(-xa, xa, 1.0f));
+  const float Lb = lg2_approx(__fmaf_rn(-xb, xb, 1.0f));
+  const unsigned long long Lp = pack_f32x2(La, Lb);
+  unsigned long long b = __float_as_uint(unit_central[COPES_NORMAL_CENTRAL_DEGREE]);
+  unsigned long long acc = (b << 32) | b;
+#pragma unroll
+  for (int k = COPES_NORMAL_CENTRAL_DEGREE - 1; k >= 0; --k) {
+    b = __float_as_uint(unit_central[k]);
+    acc = fma_f32x2(acc, Lp, (b << 32) | b);
+  }
+  float ra, rb;
+  unpack_f32x2(acc, ra, rb);
+  if (__any_sync(__activemask(), fminf(La, Lb) < COPES_NORMAL_L_SPLIT)) {
+    if (La < COPES_NORMAL_L_SPLIT) ra = tail_ratio(unit_tail, La);
+    if (Lb < COPES_NORMAL_L_SPLIT) rb = tail_ratio(unit_tail, Lb);
+  }
+  ea = __fmul_rn(xa, ra);
+  eb = __fmul_rn(xb, rb);
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t *>(&v);
