@@ -324,15 +324,19 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
   }
 }
 
-// Resident blocks per SM of the tile update: 3 x 256 threads leaves 80 registers a thread,
-// enough for G = 4 groups of Philox state, the accumulators and one noise vector's round
-// keys without spilling (measured ~5% faster than 4 blocks at 64 registers).
+// Resident blocks per SM of the tile update, by the number of noise vectors.  With many,
+// the kernel is ALU-bound: 3 x 256 threads leave 80 registers a thread for G = 4 groups of
+// Philox state, the accumulators and one noise vector's round keys (measured 5% faster
+// than 4 blocks at P = 16).  With few, the master traffic weighs more and the extra
+// resident warps hide it better: 4 blocks (measured 7% faster at P = 4).
 constexpr int kUpdateBlocksPerSM = 3;
+constexpr int kUpdateBlocksPerSMFewNoise = 4;
+constexpr int kFewNoise = 8;  // P <= kFewNoise takes the second configuration
 
 // One block per tile; the prologue folds the members into noise weights and expands each
 // noise vector's Philox round keys into shared memory.
-template <typename WT, int G, bool COMMIT>
-__global__ void __launch_bounds__(kThreads, kUpdateBlocksPerSM) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
+template <typename WT, int G, bool COMMIT, int BLOCKS>
+__global__ void __launch_bounds__(kThreads, BLOCKS) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
   __shared__ float s_w[COPES_MAX_NOISE];
   __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
   noise_weights_to_smem(a, s_w, s_rk);
@@ -419,7 +423,10 @@ template <typename WT, bool COMMIT>
 static cudaError_t launch_update_typed(int kind, const UpdateArgs &a, cudaStream_t s) {
   if (kind == COPES_SUBSPACE_TILES) {
     if (a.n_tiles == 0) return cudaSuccess;
-    update_tiles_kernel<WT, 4, COMMIT><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+    if (a.n_noise <= kFewNoise)
+      update_tiles_kernel<WT, 4, COMMIT, kUpdateBlocksPerSMFewNoise><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+    else
+      update_tiles_kernel<WT, 4, COMMIT, kUpdateBlocksPerSM><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
   } else {
     if (a.n_index == 0) return cudaSuccess;
     const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
