@@ -54,8 +54,8 @@ FALLBACK_HBM_GBS = 6800.0
 # ncu DRAM bytes per element of the dominant kernel (perturb, bf16) from one capture; the
 # figure is dropped (traffic = null) when es_kernels.cu no longer matches the hash it
 # was taken on.
-NCU_TRAFFIC = {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "7609a99dea5c3974",
-               "bytes_per_elem": 5.421, "capture": "profiles/perturb_4b_slice.md"}
+NCU_TRAFFIC = {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "fd276ea14451ff07",
+               "bytes_per_elem": 5.414, "capture": "profiles/perturb_4b_slice.md"}
 
 
 def parse():
