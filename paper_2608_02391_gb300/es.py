@@ -11,6 +11,8 @@ sync_step          one CoPES training step (Algorithm 1): every subspace's N_k =
 backup_visit       round_robin_visit in the CPU weight backup mode (Supp. A.8): the
                    context is saved to pinned host memory, members are perturbed from
                    it, and restore copies it back; no fp32 master.
+state_dict /       the resumable state (fp32 master, ES configuration, next iteration):
+load_state         noise is counter-based, so resuming from it is bit-exact.
 population_visit   round_robin_visit with the population split across the ranks of a
                    process group, each rank holding a full replica of theta: a rank
                    evaluates its slice of the members, the N reward scalars are
@@ -208,3 +210,25 @@ def population_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iter
     coef = copes.step_coef(cfg.alpha, N, s_k, cfg.convention)
     copes.update(arena, sub, nid, sign, f, seeds, coef, fuse_commit=True)
     return f
+
+
+# ------------------------------------------------------------------ checkpoint / resume
+def state_dict(arena: copes.Arena, cfg: ESConfig, next_iteration: int, **extra) -> dict:
+    """The resumable ES state: the fp32 master (host copy), the configuration and the next
+    iteration index.  Member seeds and noise are functions of (base seed, iteration,
+    subspace, member) and (seed, index), and partition seeds are part of `extra`, so
+    nothing else needs saving: a run resumed from this state continues bit for bit."""
+    return {"master": arena.master.detach().cpu().clone(), "working_dtype": str(arena.w.dtype),
+            "config": dict(cfg.__dict__), "next_iteration": int(next_iteration), **extra}
+
+
+def load_state(state: dict, device="cuda") -> tuple:
+    """Rebuilds (arena, cfg, next_iteration) from state_dict's output: the master is
+    copied to the device and the working weights are committed from it (w = round(theta)
+    over the whole arena)."""
+    master = state["master"].to(device).contiguous()
+    dtype = {"torch.bfloat16": torch.bfloat16, "torch.float32": torch.float32}[state["working_dtype"]]
+    arena = copes.Arena(torch.empty(master.numel(), dtype=dtype, device=device), master)
+    everything = copes.tiles_from_ranges([(0, master.numel())], device=device)
+    copes.context_commit(arena, everything)
+    return arena, ESConfig(**state["config"]), state["next_iteration"]
