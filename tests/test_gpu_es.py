@@ -274,3 +274,42 @@ def test_gathered_master_equals_master_path(copes, dtype):
     assert np.array_equal(s2.gathered.cpu().numpy().view(np.uint32),
                           a1.master.cpu().numpy()[inside].view(np.uint32))
     copes.check()
+
+
+def test_maximum_tile_size(copes):
+    """Tiles of COPES_TILE_MAX elements (the largest a tile table may hold) over a ragged
+    range: perturb, restore and update against the oracle at sampled elements, with the
+    range edges included; a larger tile size is rejected on the host."""
+    n = (1 << 21) + 4101
+    lo, hi = 3, n - 2
+    theta = theta_np(n, seed=12)
+    arena = make(copes, torch.bfloat16, theta)
+    before = w_bits(arena).copy()
+    sub = copes.tiles_from_ranges([(lo, hi)], tile_size=copes.TILE_MAX)
+    assert sub.tensor.shape[0] == 3
+    with pytest.raises(copes.CopesError) as e:
+        copes.tiles_from_ranges([(lo, hi)], tile_size=copes.TILE_MAX + 1)
+    assert e.value.code == copes.ERR_SIZE
+    rng = np.random.default_rng(13)
+    g = np.unique(np.concatenate([[lo, lo + 1, (1 << 20) + lo - 1, (1 << 20) + lo, hi - 2, hi - 1],
+                                  rng.integers(lo, hi, 20_000)])).astype(np.uint64)
+    copes.perturb(arena, sub, 77, 1.5e-3)
+    got = w_bits(arena)
+    ref, _ = oracle.perturb_at(g, theta[g.astype(np.int64)], 77, 1.5e-3, oracle.BF16)
+    scale = np.maximum(np.abs(theta[g.astype(np.int64)]), np.abs(np.float32(1.5e-3) * oracle.noise(77, g)))
+    assert_bf16_close(got[g.astype(np.int64)], ref.astype(np.uint16), scale)
+    assert np.array_equal(got[:lo], before[:lo]) and np.array_equal(got[hi:], before[hi:])
+    copes.restore(arena, sub)
+    assert np.array_equal(w_bits(arena)[lo:hi], oracle.bf16_bits_array(theta[lo:hi]))
+    nid, sign, P = copes.member_table(32, copes.ANTITHETIC)
+    rewards = np.linspace(0, 1, 32).astype(np.float32)
+    f = copes.shape_fitness(torch.from_numpy(rewards).cuda(), copes.SHAPE_ZSCORE)
+    seeds = copes.member_seeds(33, 0, 0, P)
+    copes.update(arena, sub, nid, sign, f, seeds, 0.01)
+    f_ref = oracle.shape_fitness(rewards, oracle.SHAPE_ZSCORE)
+    wj = oracle.noise_weights(nid, sign, f_ref, P)
+    _, exact, scl = oracle.update_at(g, theta[g.astype(np.int64)], seeds, wj, np.float32(0.01))
+    m = arena.master.cpu().numpy()
+    assert_update_close(m[g.astype(np.int64)], exact, scl)
+    assert np.array_equal(m[:lo], theta[:lo]) and np.array_equal(m[hi:], theta[hi:])
+    copes.check()
