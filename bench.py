@@ -24,7 +24,8 @@ GPU, the context in pinned host memory, no fp32 master.
 
 `--case 4b-hash` times the non-contiguous workload instead: the same 4B set split by a
 per-element hash into K = 16 subspaces, N = 64 antithetic members, one step = one sweep
-over the 16 subspaces, with the subspaces replayed from the partition seed (default) or
+over the 16 subspaces, with the subspaces replayed from the partition seed (default;
+`--hash-mode replay-mask` hashes once per visit into a membership mask) or
 read from int64 index lists (`--hash-mode lists`), or read from index lists with each
 subspace's theta kept in list order (`--hash-mode gathered`).
 
@@ -75,9 +76,10 @@ def parse():
                          "4b-hash-slice: the same on 268M parameters, for profiling; "
                          "4b-backup: the 4B step in the CPU weight backup mode (no fp32 master); "
                          "4b-sync: Algorithm 1 on the 4B set (K=4 random chunks resampled each step)")
-    ap.add_argument("--hash-mode", default="replay", choices=["replay", "lists", "gathered"],
-                    help="4b-hash: subspaces replayed from the partition seed, int64 index lists, or "
-                         "index lists with a gathered (list-order) master per subspace")
+    ap.add_argument("--hash-mode", default="replay", choices=["replay", "replay-mask", "lists", "gathered"],
+                    help="4b-hash: subspaces replayed from the partition seed (hashing in every kernel, "
+                         "or once per visit into a membership mask), int64 index lists, or index lists "
+                         "with a gathered (list-order) master per subspace")
     return ap.parse_args()
 
 
@@ -415,8 +417,11 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
     layout = copes.Layout(wl.numel, list(range(len(wl.tensors))))
     d = wl.d
     arena = make_arena(copes, torch, wl, layout)
-    if args.hash_mode == "replay":
+    mask_buf = None
+    if args.hash_mode in ("replay", "replay-mask"):
         subs = copes.hash_replay_partition(layout, wl.K, wl.partition_seed)
+        if args.hash_mode == "replay-mask":  # one mask buffer, rebuilt at every visit
+            mask_buf = torch.empty(int(subs[0].replay.n_replay_tiles) * 512, dtype=torch.int32, device="cuda")
     else:
         subs = copes.hash_partition(layout, wl.K, wl.partition_seed)
         if args.hash_mode == "gathered":  # each subspace's theta in list order (contiguous reads)
@@ -429,6 +434,8 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
 
     def step(s, events=None):
         for k in range(wl.K):
+            if mask_buf is not None:
+                es._timed(events, "mask", lambda: copes.hash_replay_mask(arena, subs[k], mask_buf))
             es.round_robin_visit(arena, subs[k], k, s, cfg, d, rewards[s * wl.K + k], fitness_out=fitness,
                                  events=events)
 
@@ -462,7 +469,7 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
     sm_mhz = clk["sm_mhz"] or float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12
     P = wl.n_members // 2
-    replay = args.hash_mode == "replay"
+    replay = args.hash_mode == "replay"  # the membership hash runs inside every kernel
     # algorithmic work of one update launch: 28 lane-ops per normal, P normals per member;
     # replay adds the membership hash of every element (one Philox call = 80 ops per 4)
     upd_ops = 28.0 * P * mean_dk + (20.0 * d if replay else 0.0)
@@ -497,6 +504,8 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
         "e2e": None,
         "gpu_launches": sum(counts.values()),
     }
+    if "mask" in per:
+        out["kernels"]["mask"] = {"ms": per["mask"], "launches": counts["mask"]}
     print(json.dumps(out), flush=True)
 
 

@@ -110,6 +110,8 @@ typedef struct {
   uint64_t seed;           /* HASH_REPLAY: the partition seed                             */
   float *gathered;         /* INDICES, optional: device fp32 [n_index], the subspace's master
                               values in list order (see copes_gather_master); NULL: none */
+  uint32_t *replay_mask;   /* HASH_REPLAY, optional: device membership bits filled by
+                              copes_hash_replay_mask; NULL: membership is hashed */
 } copes_subspace;
 
 /* Parameter layout: the model's tensors in order. */
@@ -279,6 +281,15 @@ int copes_scatter_master(const copes_params *p, const copes_subspace *S, cudaStr
  * list of (K, seed, k).  The table does not depend on K, seed or k, so the K subspaces of
  * one partition may share one table. */
 size_t copes_hash_replay_bytes(const copes_layout_desc *layout);
+
+/* Membership mask of a HASH_REPLAY subspace (a cache of its replay, no counterpart in the
+ * paper): one bit per element, 2,048 bytes per 16,384-element hash tile
+ * (S->n_replay_tiles * 2048 bytes, 16-byte aligned, in S->replay_mask, caller-owned).
+ * Hashes every element once and writes the bits of subspace S->k; afterwards the ES steps
+ * over S read the bits instead of hashing.  Meant to be built at the start of a visit and
+ * reused by its perturbs, restore and update; rebuild it when S's partition (K, k, seed)
+ * or table changes.  Asynchronous. */
+int copes_hash_replay_mask(const copes_params *p, const copes_subspace *S, cudaStream_t stream);
 int copes_hash_replay_subspace(const copes_layout_desc *layout, int K, uint64_t seed, int k,
                                void *table, size_t table_bytes, cudaStream_t stream,
                                copes_subspace *out);

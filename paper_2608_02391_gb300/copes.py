@@ -50,7 +50,7 @@ class Subspace(ctypes.Structure):
                 ("index", ctypes.c_void_p), ("n_index", ctypes.c_uint64),
                 ("replay", ctypes.c_void_p), ("n_replay_tiles", ctypes.c_uint64),
                 ("n_replay_tensors", ctypes.c_int), ("K", ctypes.c_int), ("k", ctypes.c_int),
-                ("seed", ctypes.c_uint64), ("gathered", ctypes.c_void_p)]
+                ("seed", ctypes.c_uint64), ("gathered", ctypes.c_void_p), ("replay_mask", ctypes.c_void_p)]
 
 
 class BackupParams(ctypes.Structure):
@@ -98,6 +98,7 @@ SIGNATURES = {
     "copes_update": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _F32, _I32, _VP]),
     "copes_init_normal": (_I32, [_VP, _VP, _U64, _F32, _F32, _VP]),
     "copes_gather_master": (_I32, [_VP, _VP, _VP]),
+    "copes_hash_replay_mask": (_I32, [_VP, _VP, _VP]),
     "copes_scatter_master": (_I32, [_VP, _VP, _VP]),
     "copes_backup_save": (_I32, [_VP, _VP, _VP]),
     "copes_backup_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
@@ -228,6 +229,7 @@ class SubspaceHandle:
     numel: int
     replay: Optional[Subspace] = None
     gathered: Optional[torch.Tensor] = None  # INDICES: theta in list order (gather_master)
+    mask: Optional[torch.Tensor] = None      # HASH_REPLAY: membership bits (hash_replay_mask)
 
     def struct(self) -> Subspace:
         if self.kind == SUBSPACE_HASH_REPLAY:
@@ -374,6 +376,28 @@ def gather_master(arena: Arena, sub: SubspaceHandle, stream=None) -> torch.Tenso
     S = sub.struct()
     _check(load().copes_gather_master(ctypes.byref(arena.params), ctypes.byref(S), _stream(stream)))
     return sub.gathered
+
+
+def hash_replay_mask(arena: Arena, sub: SubspaceHandle, buffer: Optional[torch.Tensor] = None,
+                     stream=None) -> torch.Tensor:
+    """copes_hash_replay_mask: hashes every element once and stores the membership bits
+    of the replay subspace `sub`; its ES steps then read them instead of hashing.  `buffer`
+    (int32, n_replay_tiles * 512) may be shared by the subspaces visited one at a time."""
+    assert sub.kind == SUBSPACE_HASH_REPLAY
+    words = int(sub.replay.n_replay_tiles) * 512
+    if buffer is None:
+        buffer = torch.empty(words, dtype=torch.int32, device=sub.tensor.device)
+    assert buffer.dtype == torch.int32 and buffer.numel() >= words
+    sub.mask = buffer
+    sub.replay.replay_mask = buffer.data_ptr()
+    _check(load().copes_hash_replay_mask(ctypes.byref(arena.params), ctypes.byref(sub.replay), _stream(stream)))
+    return buffer
+
+
+def drop_replay_mask(sub: SubspaceHandle) -> None:
+    """Back to hashing membership in every kernel."""
+    sub.mask = None
+    sub.replay.replay_mask = None
 
 
 def scatter_master(arena: Arena, sub: SubspaceHandle, stream=None) -> None:

@@ -54,6 +54,10 @@ int check_subspace(const copes_subspace *S, const char *who) {
   if (!S) return fail(COPES_ERR_INVALID_ARG, "%s: subspace is NULL", who);
   if (S->gathered && S->kind != COPES_SUBSPACE_INDICES)
     return fail(COPES_ERR_INVALID_ARG, "%s: a gathered master needs an INDICES subspace", who);
+  if (S->replay_mask && S->kind != COPES_SUBSPACE_HASH_REPLAY)
+    return fail(COPES_ERR_INVALID_ARG, "%s: a replay mask needs a HASH_REPLAY subspace", who);
+  if (!aligned(S->replay_mask, 16))
+    return fail(COPES_ERR_ALIGNMENT, "%s: replay_mask must be 16-byte aligned", who);
   if (!aligned(S->gathered, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: gathered must be 16-byte aligned", who);
   if (S->kind == COPES_SUBSPACE_TILES) {
     if (S->n_tiles && !S->tiles) return fail(COPES_ERR_INVALID_ARG, "%s: tiles is NULL", who);
@@ -103,6 +107,7 @@ copes::ReplayArgs replay_args(const copes_subspace *S) {
   r.lo = (uint32_t)lo;
   r.width = r.all ? 0u : (uint32_t)(hi - lo);
   copes::philox_round_keys(r.seed_lo, r.seed_hi, r.rk);
+  r.mask = S->replay_mask;
   return r;
 }
 
@@ -527,6 +532,18 @@ int copes_restore(const copes_params *p, const copes_subspace *S, cudaStream_t s
 
 int copes_context_commit(const copes_params *p, const copes_subspace *S, cudaStream_t stream) {
   return run_elementwise(copes::kOpRestore, p, S, 0, 0, 0.0f, 0.0f, stream, "copes_context_commit");
+}
+
+int copes_hash_replay_mask(const copes_params *p, const copes_subspace *S, cudaStream_t stream) {
+  const char *who = "copes_hash_replay_mask";
+  int rc = check_params(p, who);
+  if (rc) return rc;
+  if ((rc = check_subspace(S, who))) return rc;
+  if (S->kind != COPES_SUBSPACE_HASH_REPLAY || !S->replay_mask)
+    return fail(COPES_ERR_INVALID_ARG, "%s: needs a HASH_REPLAY subspace with replay_mask set", who);
+  copes::ReplayArgs r = replay_args(S);
+  r.mask = nullptr;  // the kernel hashes
+  return launch_status(copes::launch_replay_mask(r, p->n_alloc, S->replay_mask, stream), who);
 }
 
 int copes_gather_master(const copes_params *p, const copes_subspace *S, cudaStream_t stream) {

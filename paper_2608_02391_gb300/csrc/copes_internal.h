@@ -184,11 +184,13 @@ struct ReplayArgs {
   uint32_t lo, width;
   int all;
   uint32_t rk[20];  // Philox round keys of the partition seed
+  const uint32_t *mask;  // membership bits (copes_hash_replay_mask), or NULL: hash
 };
 cudaError_t launch_replay_elementwise(int op, int dtype, const ElemArgs &a, const ReplayArgs &r,
                                       cudaStream_t s);
 cudaError_t launch_replay_update(int dtype, const UpdateArgs &a, const ReplayArgs &r,
                                  cudaStream_t s);
+cudaError_t launch_replay_mask(const ReplayArgs &r, uint64_t n_alloc, uint32_t *mask, cudaStream_t s);
 
 // CPU weight backup mode: `backup` is the device-accessible pointer of pinned host memory.
 enum BackupOp { kBackupSave = 0, kBackupPerturb = 1, kBackupRestore = 2 };

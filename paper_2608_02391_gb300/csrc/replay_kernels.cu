@@ -3,8 +3,9 @@
 // read from a stored index list.  Each block takes 4 consecutive 16,384-element hash
 // tiles; each warp streams through its 2,048-element stretch of every tile (replay_stream):
 //  - it hashes 32 four-element groups at a time -- one Philox4x32-10 call per group at
-//    counter (e >> 2, tensor id, TAG_PARTITION), bucket floor(x K / 2^32) per word -- and
-//    appends the members of subspace k to its shared-memory buffer;
+//    counter (e >> 2, tensor id, TAG_PARTITION), bucket floor(x K / 2^32) per word, or,
+//    when the subspace carries a membership mask built once per visit, reads their bits --
+//    and appends the members of subspace k to its shared-memory buffer;
 //  - whenever the buffer holds a full batch, the warp processes it one member per lane,
 //    exactly as the gather kernels process an index list: perturb / restore / commit /
 //    init, or the fused update regenerating the P normals of each element.
@@ -25,6 +26,8 @@ constexpr int kReplayTilesPerBlock = 4;      // consecutive hash tiles per block
 static_assert(kReplayTile % 4 == 0 && kReplayTile <= 65536, "tile offsets fit 16 bits");
 constexpr int kReplayWarpGroups = kReplayTile / 4 / (kThreads / 32);  // groups per warp per tile
 constexpr int kReplayIters = kReplayWarpGroups / 32;                  // 32 groups per iteration
+
+constexpr uint64_t kMaskWordsPerTile = kReplayTile / 32;  // membership mask: one bit per element
 
 struct ReplayTile {
   uint64_t g0;        // global index of the tile's first element
@@ -87,14 +90,23 @@ __device__ __forceinline__ void replay_stream(const ReplayArgs &r, uint64_t n_al
   int pending = 0;  // warp-uniform
   // One iteration: the warp hashes 32 groups (128 elements, one group per lane) and
   // appends their members with one ballot per word slot; FULL drops the tile-end check.
-  auto iteration = [&](const ReplayTile &t, uint32_t tag, uint32_t q_lo0, uint32_t q_hi, uint32_t e,
-                       auto full) {
-    uint32_t x[4];
-    philox4x32_10_rk(q_lo0 + (e >> 2), q_hi, t.tensor_id, COPES_TAG_PARTITION, r.rk, x);
+  auto iteration = [&](const ReplayTile &t, uint64_t tile, uint32_t tag, uint32_t q_lo0, uint32_t q_hi,
+                       uint32_t e, auto full) {
+    uint32_t nib;  // membership of the group's 4 elements
+    if (r.mask) {
+      nib = (r.mask[tile * kMaskWordsPerTile + (e >> 5)] >> (e & 31u)) & 0xFu;
+    } else {
+      uint32_t x[4];
+      philox4x32_10_rk(q_lo0 + (e >> 2), q_hi, t.tensor_id, COPES_TAG_PARTITION, r.rk, x);
+      nib = 0;
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        // floor(x K / 2^32) == k  <=>  lo <= x < lo + width  (r.lo, r.width from the host)
+        nib |= ((r.all || x[i] - r.lo < r.width) && (decltype(full)::value || e + i < t.len)) ? (1u << i) : 0u;
+    }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      // floor(x K / 2^32) == k  <=>  lo <= x < lo + width  (r.lo, r.width from the host)
-      const bool m = (r.all || x[i] - r.lo < r.width) && (decltype(full)::value || e + i < t.len);
+      const bool m = (nib >> i) & 1u;
       const uint32_t bal = __ballot_sync(0xffffffffu, m);
       if (m) wbuf[pending + __popc(bal & lt)] = tag | (e + i);
       pending += __popc(bal);
@@ -124,10 +136,10 @@ __device__ __forceinline__ void replay_stream(const ReplayArgs &r, uint64_t n_al
     const uint32_t e0 = warp * (4u * kReplayWarpGroups) + 4u * lane;  // this lane's first group
     if (t.len == (uint32_t)kReplayTile) {
       for (int it = 0; it < kReplayIters; ++it)
-        iteration(t, tag, q_lo0, q_hi, e0 + 128u * it, std::true_type{});
+        iteration(t, tile, tag, q_lo0, q_hi, e0 + 128u * it, std::true_type{});
     } else if (t.len > 0) {
       for (int it = 0; it < kReplayIters; ++it)
-        iteration(t, tag, q_lo0, q_hi, e0 + 128u * it, std::false_type{});
+        iteration(t, tile, tag, q_lo0, q_hi, e0 + 128u * it, std::false_type{});
     }
   }
   // pool the leftovers and process them with the whole block
@@ -252,6 +264,40 @@ __global__ void __launch_bounds__(kThreads) replay_update_kernel(const __grid_co
 
 static unsigned replay_blocks(uint64_t n_tiles) {
   return (unsigned)((n_tiles + kReplayTilesPerBlock - 1) / kReplayTilesPerBlock);
+}
+
+// Membership mask of subspace r.k: bit (e mod 32) of word tile * 512 + e / 32 is set when
+// element e of hash tile `tile` belongs to it.  One block per hash tile; each lane hashes
+// one group per step and 8 lanes' 4-bit nibbles make a word.  Tiles the table maps outside
+// the arena are flagged and written as empty.
+__global__ void __launch_bounds__(kThreads) replay_mask_kernel(const __grid_constant__ ReplayArgs r,
+                                                               uint64_t n_alloc, uint32_t *mask) {
+  const uint64_t tile = blockIdx.x;
+  const ReplayTile t = replay_tile(r, n_alloc, tile);
+  const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
+  const uint32_t q_lo0 = (uint32_t)t.q0, q_hi = (uint32_t)(t.q0 >> 32);
+  for (int it = 0; it < kReplayIters; ++it) {
+    const uint32_t e = warp * (4u * kReplayWarpGroups) + 128u * it + 4u * lane;
+    uint32_t nib = 0;
+    if (e < t.len) {
+      uint32_t x[4];
+      philox4x32_10_rk(q_lo0 + (e >> 2), q_hi, t.tensor_id, COPES_TAG_PARTITION, r.rk, x);
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+        nib |= ((r.all || x[i] - r.lo < r.width) && e + i < t.len) ? (1u << i) : 0u;
+    }
+    uint32_t word = nib << (4u * (lane & 7u));
+    word |= __shfl_xor_sync(0xffffffffu, word, 1);
+    word |= __shfl_xor_sync(0xffffffffu, word, 2);
+    word |= __shfl_xor_sync(0xffffffffu, word, 4);
+    if ((lane & 7u) == 0) mask[tile * kMaskWordsPerTile + (e >> 5)] = word;
+  }
+}
+
+cudaError_t launch_replay_mask(const ReplayArgs &r, uint64_t n_alloc, uint32_t *mask, cudaStream_t s) {
+  if (r.n_tiles == 0) return cudaSuccess;
+  replay_mask_kernel<<<(unsigned)r.n_tiles, kThreads, 0, s>>>(r, n_alloc, mask);
+  return cudaGetLastError();
 }
 
 template <int OP, typename WT>

@@ -233,3 +233,17 @@ def test_gathered_master_arguments_are_rejected_before_any_launch(lib):
     idx.gathered = fake + 4
     assert lib.copes_gather_master(ctypes.byref(p), ctypes.byref(idx), None) == copes.ERR_ALIGNMENT
     assert lib.copes_restore(ctypes.byref(p), ctypes.byref(idx), None) == copes.ERR_ALIGNMENT
+
+
+def test_replay_mask_arguments_are_rejected_before_any_launch(lib):
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    p = copes.Params(fake, fake, 100, copes.BF16)
+    tiles = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
+    tiles.replay_mask = fake
+    assert lib.copes_perturb(ctypes.byref(p), ctypes.byref(tiles), 1, 1e-3, None) == copes.ERR_INVALID_ARG
+    S = copes.Subspace(kind=copes.SUBSPACE_HASH_REPLAY, replay=fake, n_replay_tiles=2, n_replay_tensors=1,
+                       K=4, k=1, seed=7)
+    assert lib.copes_hash_replay_mask(ctypes.byref(p), ctypes.byref(S), None) == copes.ERR_INVALID_ARG
+    S.replay_mask = fake + 4
+    assert lib.copes_hash_replay_mask(ctypes.byref(p), ctypes.byref(S), None) == copes.ERR_ALIGNMENT

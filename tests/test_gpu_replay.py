@@ -177,3 +177,36 @@ def test_table_past_the_arena_is_skipped_and_reported(copes, layout):
     outside[g[g < 60_000]] = False
     assert np.array_equal(got[outside], before[outside])
     copes.check()
+
+
+@pytest.mark.parametrize("K,k", [(1, 0), (16, 5), (64, 63), (3, 2)])
+def test_membership_mask_equals_hashing(copes, layout, K, k):
+    """A replay subspace with its membership mask gives the hashing path's results bit for
+    bit: perturb, restore, update (fused commit)."""
+    n = layout.d_pad
+    theta = theta_np(n, seed=K)
+    a1, a2 = make(copes, torch.bfloat16, theta), make(copes, torch.bfloat16, theta)
+    s1 = copes.hash_replay_partition(layout, K, PSEED, count=False)[k]
+    s2 = copes.hash_replay_partition(layout, K, PSEED, count=False)[k]
+    mask = copes.hash_replay_mask(a2, s2)
+    # the mask holds exactly the oracle's members
+    bits = np.unpackbits(mask.cpu().numpy().view(np.uint8), bitorder="little").astype(bool)
+    assert bits.sum() == oracle.hash_list(NUMEL, TIDS, K, PSEED, k).size
+    for seed, ss in [(3, 1e-3), (4, -2e-3)]:
+        copes.perturb(a1, s1, seed, ss)
+        copes.perturb(a2, s2, seed, ss)
+        assert np.array_equal(w_bits(a1), w_bits(a2))
+    copes.restore(a1, s1)
+    copes.restore(a2, s2)
+    nid, sign, P = copes.member_table(32, copes.ANTITHETIC)
+    f = torch.linspace(-1, 1, 32, device="cuda")
+    seeds = copes.member_seeds(33, 0, k, P)
+    copes.update(a1, s1, nid, sign, f, seeds, 0.2)
+    copes.update(a2, s2, nid, sign, f, seeds, 0.2)
+    assert np.array_equal(w_bits(a1), w_bits(a2))
+    assert torch.equal(a1.master.view(torch.int32), a2.master.view(torch.int32))
+    copes.drop_replay_mask(s2)
+    copes.perturb(a2, s2, 5, 1e-3)
+    copes.perturb(a1, s1, 5, 1e-3)
+    assert np.array_equal(w_bits(a1), w_bits(a2))
+    copes.check()
