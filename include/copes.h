@@ -92,9 +92,10 @@ typedef struct {
  *               gather form used for hash partitions).  The array must be 16-byte aligned.
  *  HASH_REPLAY: subspace k of the HASH partition (K, seed), with membership recomputed
  *               from the partition seed inside every kernel instead of read from a list
- *               (Supp. A.8 "Partition Replay").  Same members as the INDICES list that
- *               copes_hash_fill writes for (K, seed, k).  Filled by
- *               copes_hash_replay_subspace; `replay` is a device tensor table it writes. */
+ *               (Supp. A.8 "Partition Replay"), or read from its optional membership
+ *               mask.  Same members as the INDICES list that copes_hash_fill writes for
+ *               (K, seed, k).  Filled by copes_hash_replay_subspace; `replay` is a device
+ *               tensor table it writes. */
 enum { COPES_SUBSPACE_TILES = 0, COPES_SUBSPACE_INDICES = 1, COPES_SUBSPACE_HASH_REPLAY = 2 };
 typedef struct {
   int kind;
@@ -277,10 +278,14 @@ int copes_scatter_master(const copes_params *p, const copes_subspace *S, cudaStr
  * asynchronous copies on `stream`, and fills *out as the HASH_REPLAY subspace k of the
  * partition (K, seed).  No list is built: perturb, restore, commit and update over *out
  * recompute, per 16,384-element tile, each element's bucket floor(x K / 2^32) (x as in
- * copes_hash_count), gather the members of subspace k in shared memory and process them.  Results are identical to those over the INDICES
- * list of (K, seed, k).  The table does not depend on K, seed or k, so the K subspaces of
- * one partition may share one table. */
+ * copes_hash_count), gather the members of subspace k in shared memory and process them.
+ * Results are identical to those over the INDICES list of (K, seed, k).  The table does
+ * not depend on K, seed or k, so the K subspaces of one partition may share one table. */
 size_t copes_hash_replay_bytes(const copes_layout_desc *layout);
+
+int copes_hash_replay_subspace(const copes_layout_desc *layout, int K, uint64_t seed, int k,
+                               void *table, size_t table_bytes, cudaStream_t stream,
+                               copes_subspace *out);
 
 /* Membership mask of a HASH_REPLAY subspace (a cache of its replay, no counterpart in the
  * paper): one bit per element, 2,048 bytes per 16,384-element hash tile
@@ -290,9 +295,6 @@ size_t copes_hash_replay_bytes(const copes_layout_desc *layout);
  * reused by its perturbs, restore and update; rebuild it when S's partition (K, k, seed)
  * or table changes.  Asynchronous. */
 int copes_hash_replay_mask(const copes_params *p, const copes_subspace *S, cudaStream_t stream);
-int copes_hash_replay_subspace(const copes_layout_desc *layout, int K, uint64_t seed, int k,
-                               void *table, size_t table_bytes, cudaStream_t stream,
-                               copes_subspace *out);
 
 /* ------------------------------------------------------------------------- ES steps */
 
