@@ -69,6 +69,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
+    ap.add_argument("--cpu-cores", type=int, default=0,
+                    help="processes of the oracle's CPU sample (0: every core this process may use)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice", "4b-backup", "4b-sync"],
                     help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling; "
@@ -175,17 +177,19 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------------ CPU oracle leg
-def oracle_visit_sample(wl, n_sample: int, iteration: int = 0):
+def oracle_visit_sample(wl, n_sample: int, iteration: int = 0, part: int = 0):
     """The oracle as it stands on a bounded sample: one subspace visit (N perturbs,
-    restore, shaping, fused update + commit) restricted to the first n_sample parameters
-    of subspace 0.  Returns (seconds, parameters)."""
+    restore, shaping, fused update + commit) restricted to parameters
+    [part * n_sample, (part + 1) * n_sample) of subspace 0.  Returns (seconds, parameters)."""
     import oracle
     from paper_2608_02391_gb300 import workloads
     N = wl.n_members
-    rng = np.random.default_rng(0)
-    master = (rng.standard_normal(n_sample) * 0.02).astype(np.float32)
-    w = np.zeros(n_sample, np.uint16)
-    sub = oracle.make_subspace(ranges=[(0, n_sample)])
+    b = part * n_sample
+    rng = np.random.default_rng(part)
+    master = np.zeros(b + n_sample, np.float32)  # pages below b are never touched
+    master[b:] = rng.standard_normal(n_sample) * 0.02
+    w = np.zeros(b + n_sample, np.uint16)
+    sub = oracle.make_subspace(ranges=[(b, b + n_sample)])
     nid, sign, P = oracle.member_table(N, oracle.ANTITHETIC)
     seeds = np.array([oracle.member_seed(wl.base_seed, iteration, 0, j) for j in range(P)], np.uint64)
     rewards = workloads.reward_stream(wl, 1)[0]
@@ -199,29 +203,71 @@ def oracle_visit_sample(wl, n_sample: int, iteration: int = 0):
     return time.perf_counter() - t0, n_sample
 
 
+def _oracle_part(args):
+    return oracle_visit_sample(*args)
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+class OraclePool:
+    """The oracle on every host core: one spawned process per core (spawn, not fork: the
+    parent may hold a CUDA context), each running the same visit on its own disjoint
+    range of subspace 0.  Throughput = all ranges' parameters / the wall time of the
+    parallel map."""
+
+    def __init__(self, wl, cores: int):
+        import multiprocessing as mp
+        import oracle
+        oracle.build()
+        self.wl, self.cores = wl, max(1, cores)
+        self.pool = mp.get_context("spawn").Pool(self.cores) if self.cores > 1 else None
+
+    def visit(self, n_per_core: int, iteration: int = 0):
+        jobs = [(self.wl, n_per_core, iteration, part) for part in range(self.cores)]
+        t0 = time.perf_counter()
+        res = self.pool.map(_oracle_part, jobs, chunksize=1) if self.pool else [_oracle_part(jobs[0])]
+        wall = time.perf_counter() - t0
+        return wall, sum(m for _, m in res)
+
+    def close(self):
+        if self.pool:
+            self.pool.close()
+            self.pool.join()
+
+
 def run_reference(args, wl):
     rank, world, _ = dist_env()
     if world > 1 and rank != 0:
         return
-    import oracle
-    oracle.build()
     n = max(1024, args.cpu_sample // 4)
-    for _ in range(max(args.warmup, 0)):
-        oracle_visit_sample(wl, 1024)
-    tot_t, tot_n = 0.0, 0
-    for s in range(args.steps):
-        t, m = oracle_visit_sample(wl, n, iteration=s)
-        tot_t += t
-        tot_n += m
+    pool = OraclePool(wl, args.cpu_cores or host_cores())
+    try:
+        pool.visit(1024)  # loads the oracle in every worker
+        for _ in range(max(args.warmup, 0)):
+            pool.visit(1024)
+        tot_t, tot_n = 0.0, 0
+        for s in range(args.steps):
+            t, m = pool.visit(n, iteration=s)
+            tot_t += t
+            tot_n += m
+    finally:
+        pool.close()
     value = tot_n / tot_t
     sample = (f"each step: one subspace visit (N={wl.n_members} perturbs, restore, z-score shaping, "
-              f"fused update + commit) over {n} parameters, single thread")
+              f"fused update + commit) over {n} parameters per core, {pool.cores} processes on "
+              f"disjoint ranges of subspace 0")
     print(json.dumps({
         "impl": "reference", "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot_t / args.steps,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": workload_config(wl, args),
-        "cpu_baseline": {"value": value, "unit": "params/s", "cores": 1, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": "params/s", "cores": pool.cores, "kind": "oracle",
+                         "sample": sample},
         "e2e": {"value": value, "unit": "params/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }), flush=True)
 
@@ -398,13 +444,17 @@ def main():
         "gpu_launches": launches,
     }
     if not args.no_cpu_baseline and world == 1:
-        import oracle
-        oracle.build()
-        t, m = oracle_visit_sample(wl, args.cpu_sample)
+        pool = OraclePool(wl, args.cpu_cores or host_cores())
+        try:
+            pool.visit(1024)  # loads the oracle in every worker
+            t, m = pool.visit(args.cpu_sample)
+        finally:
+            pool.close()
         out["cpu_baseline"] = {
-            "value": m / t, "unit": "params/s", "cores": 1, "kind": "oracle",
+            "value": m / t, "unit": "params/s", "cores": pool.cores, "kind": "oracle",
             "sample": f"one subspace visit (N={wl.n_members} perturbs, restore, shaping, fused update + "
-                      f"commit) over {m} parameters of subspace 0, single thread, {t:.1f} s"}
+                      f"commit) over {args.cpu_sample} parameters per core, {pool.cores} processes on "
+                      f"disjoint ranges of subspace 0 ({m} parameters), {t:.1f} s"}
     print(json.dumps(out), flush=True)
     if world > 1:
         dist.destroy_process_group()

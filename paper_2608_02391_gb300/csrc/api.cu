@@ -103,9 +103,8 @@ copes::ReplayArgs replay_args(const copes_subspace *S) {
   // floor(x K / 2^32) == k  <=>  ceil(k 2^32 / K) <= x < ceil((k + 1) 2^32 / K)
   const uint64_t lo = (((uint64_t)S->k << 32) + (uint64_t)S->K - 1) / (uint64_t)S->K;
   const uint64_t hi = (((uint64_t)(S->k + 1) << 32) + (uint64_t)S->K - 1) / (uint64_t)S->K;
-  r.all = S->K == 1;
   r.lo = (uint32_t)lo;
-  r.width = r.all ? 0u : (uint32_t)(hi - lo);
+  r.span = (uint32_t)(hi - lo - 1);
   copes::philox_round_keys(r.seed_lo, r.seed_hi, r.rk);
   r.mask = S->replay_mask;
   return r;

@@ -180,9 +180,9 @@ struct ReplayArgs {
   uint64_t n_tiles;  // hash tiles of kHashTile elements covered by the table
   uint32_t seed_lo, seed_hi;
   int K, k;
-  // bucket k is the word range [lo, lo + width): lo = ceil(k 2^32 / K); all = (K == 1)
-  uint32_t lo, width;
-  int all;
+  // bucket k is the word range [lo, lo + span] (32-bit unsigned): lo = ceil(k 2^32 / K),
+  // span = ceil((k + 1) 2^32 / K) - lo - 1 (2^32 - 1 when K = 1)
+  uint32_t lo, span;
   uint32_t rk[20];  // Philox round keys of the partition seed
   const uint32_t *mask;  // membership bits (copes_hash_replay_mask), or NULL: hash
 };

@@ -72,8 +72,10 @@ __device__ __forceinline__ ReplayTile replay_tile(const ReplayArgs &r, uint64_t 
 // per lane, every lane busy, so the hashing (ALU) interleaves with the members' scattered
 // loads and stores.  The warps' leftovers (fewer than BATCH each) are pooled and processed
 // by the whole block at the end; `flush` then runs once.  Every warp runs the same
-// iterations, so the full-warp ballots and shuffles see all 32 lanes.
-template <int BATCH, typename Fn, typename Flush>
+// iterations, so the full-warp ballots and shuffles see all 32 lanes.  MASK: membership
+// comes from r.mask (non-null) instead of the hash; a compile-time choice, so the hashing
+// variant carries no mask code.
+template <int BATCH, bool MASK, typename Fn, typename Flush>
 __device__ __forceinline__ void replay_stream(const ReplayArgs &r, uint64_t n_alloc, uint32_t *wbuf,
                                               uint64_t (*s_g0)[kReplayTilesPerBlock], uint32_t *pool,
                                               int *pool_n, Fn process, Flush flush) {
@@ -92,23 +94,23 @@ __device__ __forceinline__ void replay_stream(const ReplayArgs &r, uint64_t n_al
   // appends their members with one ballot per word slot; FULL drops the tile-end check.
   auto iteration = [&](const ReplayTile &t, uint64_t tile, uint32_t tag, uint32_t q_lo0, uint32_t q_hi,
                        uint32_t e, auto full) {
-    uint32_t nib;  // membership of the group's 4 elements
-    if (r.mask) {
-      nib = (r.mask[tile * kMaskWordsPerTile + (e >> 5)] >> (e & 31u)) & 0xFu;
+    bool m[4];  // membership of the group's 4 elements
+    if constexpr (MASK) {
+      const uint32_t nib = r.mask[tile * kMaskWordsPerTile + (e >> 5)] >> (e & 31u);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) m[i] = (nib >> i) & 1u;
     } else {
       uint32_t x[4];
       philox4x32_10_rk(q_lo0 + (e >> 2), q_hi, t.tensor_id, COPES_TAG_PARTITION, r.rk, x);
-      nib = 0;
 #pragma unroll
       for (int i = 0; i < 4; ++i)
-        // floor(x K / 2^32) == k  <=>  lo <= x < lo + width  (r.lo, r.width from the host)
-        nib |= ((r.all || x[i] - r.lo < r.width) && (decltype(full)::value || e + i < t.len)) ? (1u << i) : 0u;
+        // floor(x K / 2^32) == k  <=>  x - lo <= span in 32-bit unsigned arithmetic
+        m[i] = x[i] - r.lo <= r.span && (decltype(full)::value || e + i < t.len);
     }
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      const bool m = (nib >> i) & 1u;
-      const uint32_t bal = __ballot_sync(0xffffffffu, m);
-      if (m) wbuf[pending + __popc(bal & lt)] = tag | (e + i);
+      const uint32_t bal = __ballot_sync(0xffffffffu, m[i]);
+      if (m[i]) wbuf[pending + __popc(bal & lt)] = tag | (e + i);
       pending += __popc(bal);
     }
     __syncwarp();
@@ -169,7 +171,7 @@ constexpr uint32_t replay_tag() { return OP == kOpInit ? COPES_TAG_INIT : COPES_
 
 // Perturb / restore / commit / init over the members of the block's hash tiles: four
 // members per lane per batch, their master loads issued together.
-template <int OP, typename WT>
+template <int OP, typename WT, bool MASK>
 __global__ void __launch_bounds__(kThreads) replay_elem_kernel(const __grid_constant__ ElemArgs a,
                                                                const __grid_constant__ ReplayArgs r) {
   constexpr int BATCH = 128;
@@ -181,8 +183,8 @@ __global__ void __launch_bounds__(kThreads) replay_elem_kernel(const __grid_cons
   if (threadIdx.x == 0) s_pool_n = 0;
   __syncthreads();
   float *__restrict__ master = a.master;
-  replay_stream<BATCH>(r, a.n_alloc, s_buf[threadIdx.x >> 5], s_g0, s_pool, &s_pool_n,
-                       [&](const uint64_t (&g)[U], const bool (&ok)[U]) {
+  replay_stream<BATCH, MASK>(r, a.n_alloc, s_buf[threadIdx.x >> 5], s_g0, s_pool, &s_pool_n,
+                             [&](const uint64_t (&g)[U], const bool (&ok)[U]) {
     float th[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) th[u] = (OP != kOpInit && ok[u]) ? master[g[u]] : 0.0f;
@@ -208,7 +210,7 @@ __global__ void __launch_bounds__(kThreads) replay_elem_kernel(const __grid_cons
 
 // The fused update over the members of the block's hash tiles: two members per lane per
 // batch, each regenerating the P normals of its element.
-template <typename WT, bool COMMIT>
+template <typename WT, bool COMMIT, bool MASK>
 __global__ void __launch_bounds__(kThreads) replay_update_kernel(const __grid_constant__ UpdateArgs a,
                                                                  const __grid_constant__ ReplayArgs r) {
   constexpr int BATCH = 64;
@@ -223,8 +225,8 @@ __global__ void __launch_bounds__(kThreads) replay_update_kernel(const __grid_co
   noise_weights_to_smem(a, s_w, s_rk);  // ends with __syncthreads
   float *__restrict__ master = a.master;
   const int P = a.n_noise;
-  replay_stream<BATCH>(r, a.n_alloc, s_buf[threadIdx.x >> 5], s_g0, s_pool, &s_pool_n,
-                       [&](const uint64_t (&g)[U], const bool (&ok)[U]) {
+  replay_stream<BATCH, MASK>(r, a.n_alloc, s_buf[threadIdx.x >> 5], s_g0, s_pool, &s_pool_n,
+                             [&](const uint64_t (&g)[U], const bool (&ok)[U]) {
     float acc[U];
 #pragma unroll
     for (int u = 0; u < U; ++u) acc[u] = 0.0f;
@@ -284,7 +286,7 @@ __global__ void __launch_bounds__(kThreads) replay_mask_kernel(const __grid_cons
       philox4x32_10_rk(q_lo0 + (e >> 2), q_hi, t.tensor_id, COPES_TAG_PARTITION, r.rk, x);
 #pragma unroll
       for (int i = 0; i < 4; ++i)
-        nib |= ((r.all || x[i] - r.lo < r.width) && e + i < t.len) ? (1u << i) : 0u;
+        nib |= (x[i] - r.lo <= r.span && e + i < t.len) ? (1u << i) : 0u;
     }
     uint32_t word = nib << (4u * (lane & 7u));
     word |= __shfl_xor_sync(0xffffffffu, word, 1);
@@ -303,7 +305,10 @@ cudaError_t launch_replay_mask(const ReplayArgs &r, uint64_t n_alloc, uint32_t *
 template <int OP, typename WT>
 static cudaError_t launch_replay_elem_typed(const ElemArgs &a, const ReplayArgs &r, cudaStream_t s) {
   if (r.n_tiles == 0) return cudaSuccess;
-  replay_elem_kernel<OP, WT><<<replay_blocks(r.n_tiles), kThreads, 0, s>>>(a, r);
+  if (r.mask)
+    replay_elem_kernel<OP, WT, true><<<replay_blocks(r.n_tiles), kThreads, 0, s>>>(a, r);
+  else
+    replay_elem_kernel<OP, WT, false><<<replay_blocks(r.n_tiles), kThreads, 0, s>>>(a, r);
   return cudaGetLastError();
 }
 
@@ -326,7 +331,10 @@ cudaError_t launch_replay_elementwise(int op, int dtype, const ElemArgs &a, cons
 template <typename WT, bool COMMIT>
 static cudaError_t launch_replay_update_typed(const UpdateArgs &a, const ReplayArgs &r, cudaStream_t s) {
   if (r.n_tiles == 0) return cudaSuccess;
-  replay_update_kernel<WT, COMMIT><<<replay_blocks(r.n_tiles), kThreads, 0, s>>>(a, r);
+  if (r.mask)
+    replay_update_kernel<WT, COMMIT, true><<<replay_blocks(r.n_tiles), kThreads, 0, s>>>(a, r);
+  else
+    replay_update_kernel<WT, COMMIT, false><<<replay_blocks(r.n_tiles), kThreads, 0, s>>>(a, r);
   return cudaGetLastError();
 }
 
