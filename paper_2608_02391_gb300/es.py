@@ -11,6 +11,9 @@ sync_step          one CoPES training step (Algorithm 1): every subspace's N_k =
 backup_visit       round_robin_visit in the CPU weight backup mode (Supp. A.8): the
                    context is saved to pinned host memory, members are perturbed from
                    it, and restore copies it back; no fp32 master.
+ChunkPrefetcher    the random-chunk partition of the next sync_step built on a side stream
+                   while the current step's kernels run (Algorithm 1 resamples it every
+                   step).
 state_dict /       the resumable state (fp32 master, ES configuration, next iteration):
 load_state         noise is counter-based, so resuming from it is bit-exact.
 population_visit   round_robin_visit with the population split across the ranks of a
@@ -160,6 +163,55 @@ def build_subspaces(layout: copes.Layout, mode: str, K: int, group_of: Optional[
         return [copes.subspace_build(layout, copes.PART_RANDOM_CHUNKS, K, k, seed=seed, chunk=chunk,
                                      chunk_map=cmap, tile_size=tile_size) for k in range(K)]
     raise ValueError(mode)
+
+
+class ChunkPrefetcher:
+    """Random equal-size chunk partitions (Algorithm 1 resamples the partition every step,
+    Sec. 3.2), each built one step ahead on a side stream.
+
+    Building a partition copies the device chunk map to the host and synchronises the
+    stream it runs on before the host writes the tile tables.  On a side stream that
+    wait covers only the map's own kernels, so the host builds step s + 1's tables while
+    the main stream still executes step s, and the copy engines move them meanwhile.
+    take(s) makes the caller's stream wait for step s's build and records the tables'
+    use on that stream, so the caching allocator keeps them until its kernels are done.
+    """
+
+    def __init__(self, layout: copes.Layout, K: int, seed_of: Callable[[int], int], chunk: int = 65536,
+                 tile_size: int = copes.DEFAULT_TILE, device="cuda"):
+        self.layout, self.K, self.seed_of = layout, K, seed_of
+        self.chunk, self.tile_size = chunk, tile_size
+        self.side = torch.cuda.Stream(device=device)
+        self.ready = {}
+
+    def _build(self, step: int, events: Optional[dict] = None):
+        start = end = None
+        if events is not None:
+            start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        done = torch.cuda.Event()
+        with torch.cuda.stream(self.side):
+            if start is not None:
+                start.record(self.side)
+            subs = build_subspaces(self.layout, "random_chunks", self.K, seed=self.seed_of(step),
+                                   chunk=self.chunk, tile_size=self.tile_size)
+            if end is not None:
+                end.record(self.side)
+                events.setdefault("partition", []).append((start, end))
+            done.record(self.side)
+        return subs, done
+
+    def prefetch(self, step: int, events: Optional[dict] = None) -> None:
+        if step not in self.ready:
+            self.ready[step] = self._build(step, events)
+
+    def take(self, step: int, stream: Optional[torch.cuda.Stream] = None,
+             events: Optional[dict] = None) -> List[copes.SubspaceHandle]:
+        subs, done = self.ready.pop(step, None) or self._build(step, events)
+        stream = stream or torch.cuda.current_stream()
+        stream.wait_event(done)
+        for sub in subs:
+            sub.tensor.record_stream(stream)
+        return subs
 
 
 # ------------------------------------------------------------- population parallelism

@@ -414,3 +414,46 @@ def test_sync_step_algorithm1_matches_oracle(copes, joint):
         _, exact, scale = oracle.update_at(g, theta0[g.astype(np.int64)], seeds, wj, coef)
         assert_update_close(got[g.astype(np.int64)], exact, scale)
     copes.check()
+
+
+def test_sync_steps_with_prefetched_partitions_are_bit_identical(copes):
+    """Algorithm 1 resamples the partition every step.  Building step s + 1's partition on
+    a side stream while step s runs (es.ChunkPrefetcher) gives the oracle's chunk ranges and
+    the same three-step trajectory, bit for bit, as building each partition in line."""
+    from paper_2608_02391_gb300 import es
+    n, K, N, chunk, steps = 1 << 20, 4, 8, 4096, 3
+    theta0, _ = wl.tiny_theta_and_objective()
+    layout = copes.Layout([n])
+    cfg = es.ESConfig(n_members=N, sigma=1e-3, alpha=5e-4, shaping="zscore",
+                      convention=copes.COEF_PAPER, dimension_aware=True)
+    rewards = torch.from_numpy((np.random.default_rng(3).integers(0, 17, (steps, N)) / 16)
+                               .astype(np.float32)).cuda()
+    seed_of = lambda s: 500 + s  # noqa: E731
+
+    def run(prefetch):
+        master = torch.from_numpy(theta0.copy()).cuda()
+        arena = copes.Arena(master.to(torch.bfloat16), master)
+        parts = es.ChunkPrefetcher(layout, K, seed_of, chunk=chunk)
+        seen = []
+        for s in range(steps):
+            if prefetch:
+                subs = parts.take(s)
+            else:
+                subs = es.build_subspaces(layout, "random_chunks", K, seed=seed_of(s), chunk=chunk)
+            seen.append([tile_ranges(sub) for sub in subs])
+            es.sync_step(arena, subs, s, cfg, n, rewards[s], joint=True)
+            if prefetch and s + 1 < steps:
+                parts.prefetch(s + 1)
+        torch.cuda.synchronize()
+        return master.cpu().numpy(), arena.w.view(torch.int16).cpu().numpy(), seen
+
+    m_ref, w_ref, seen_ref = run(False)
+    m_got, w_got, seen_got = run(True)
+    for s in range(steps):
+        cmap = oracle.random_chunks(n // chunk, K, seed_of(s))
+        for k in range(K):
+            assert seen_got[s][k] == seen_ref[s][k] == oracle.chunk_ranges([n], chunk, cmap, k)
+    assert np.array_equal(m_got.view(np.uint32), m_ref.view(np.uint32))
+    assert np.array_equal(w_got, w_ref)
+    assert not np.array_equal(m_ref, theta0)
+    copes.check()
