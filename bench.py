@@ -52,11 +52,15 @@ sys.path.insert(0, ROOT)
 METRIC = "ES-iteration params/s and HBM GB/s at 4B bf16 (N=32), % of roofline on 1 GB300"
 FALLBACK_HBM_GBS = 6800.0
 
-# ncu DRAM bytes per element of the dominant kernel (perturb, bf16) from one capture; the
-# figure is dropped (traffic = null) when es_kernels.cu no longer matches the hash it
-# was taken on.
-NCU_TRAFFIC = {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "fd276ea14451ff07",
-               "bytes_per_elem": 5.414, "capture": "profiles/perturb_4b_slice.md"}
+# ncu DRAM bytes per element of the dominant kernel (the pair perturb, or the plain perturb
+# under --no-partner; bf16) from one capture each; a figure is dropped (traffic = null)
+# when es_kernels.cu or copes_device.cuh no longer matches the hash it was taken on.
+NCU_TRAFFIC = {
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "6645acd4b5b44240",
+                     "bytes_per_elem": 7.231, "capture": "profiles/perturb_pair_4b_slice.md"},
+    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "fd276ea14451ff07",
+                "bytes_per_elem": 5.414, "capture": "profiles/perturb_4b_slice.md"},
+}
 
 
 def parse():
@@ -69,6 +73,8 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
+    ap.add_argument("--no-partner", action="store_true",
+                    help="perturb every member from theta (no antithetic partner buffer)")
     ap.add_argument("--cpu-cores", type=int, default=0,
                     help="processes of the oracle's CPU sample (0: every core this process may use)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -331,6 +337,9 @@ def main():
     spec_groups = np.ascontiguousarray(wl.group_of, np.int32)
     subs = es.build_subspaces(layout, "groups", wl.K, group_of=wl.group_of, tile_size=args.tile)
     tile_buf = [s.tensor for s in subs]
+    # antithetic pairs: one noise generation per pair, the partner's weights staged in a
+    # buffer as wide as the widest subspace
+    partners = [None] * wl.K if args.no_partner else es.Partner.per_subspace(arena, subs)
 
     import ctypes
     L = copes.load()
@@ -348,7 +357,7 @@ def main():
         for k in range(wl.K):
             rebuild(k)
             es.round_robin_visit(arena, subs[k], k, s, cfg, d, rewards_dev[s * wl.K + k],
-                                 fitness_out=fitness, events=events)
+                                 fitness_out=fitness, events=events, partner=partners[k])
 
     for s in range(args.warmup):
         step(s)
@@ -384,7 +393,7 @@ def main():
             rebuild(k)
             r_dev.copy_(pinned[s * wl.K + k], non_blocking=True)
             es.round_robin_visit(arena, subs[k], k, s, cfg, d, r_dev, fitness_out=f_all[k],
-                                 events=e2e_events)
+                                 events=e2e_events, partner=partners[k])
         fit_host.copy_(f_all, non_blocking=True)
         torch.cuda.synchronize()
     e2e_s = max_over_ranks(time.perf_counter() - t0, "cuda")
@@ -400,11 +409,15 @@ def main():
     mean_dk = float(np.mean(d_k))
     peaks, peak_src = measured_peaks()
     hbm = float(peaks["hbm_gbs"])
-    perturb_bytes = 6.0 * mean_dk
+    paired = "partner" in per
+    # the pair perturb reads theta (4 B) and writes w and the partner's weights (2 + 2 B);
+    # the partner copy reads and writes 2 B; a plain perturb reads 4 B and writes 2 B
+    perturb_bytes = (8.0 if paired else 6.0) * mean_dk
     achieved = perturb_bytes / (per["perturb"] * 1e-3) / 1e9
+    ncu = NCU_TRAFFIC["perturb_pair" if paired else "perturb"]
     traffic = None
-    if NCU_TRAFFIC["source_sha"] == source_sha() and NCU_TRAFFIC["bytes_per_elem"]:
-        traffic = NCU_TRAFFIC["bytes_per_elem"] * mean_dk
+    if ncu["source_sha"] == source_sha() and ncu["bytes_per_elem"]:
+        traffic = ncu["bytes_per_elem"] * mean_dk
     props = torch.cuda.get_device_properties(local)
     clk = clocks.summary()
     n_normals_update = wl.n_members // 2
@@ -422,12 +435,12 @@ def main():
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": workload_config(wl, args),
         "hbm_gbs": bytes_per_step * args.steps / (ms * 1e-3) / 1e9,
-        "roofline": {"bound": "hbm", "kernel": "perturb", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                     "frac": achieved / hbm, "traffic": traffic, "peak_source": peak_src,
-                     "algorithmic_bytes_per_launch": perturb_bytes},
+        "roofline": {"bound": "hbm", "kernel": "perturb_pair" if paired else "perturb", "achieved": achieved,
+                     "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
+                     "peak_source": peak_src, "algorithmic_bytes_per_launch": perturb_bytes},
         "kernels": {
-            "perturb": {"ms": per["perturb"], "launches": counts["perturb"], "GB/s": achieved,
-                        "frac_hbm": achieved / hbm},
+            ("perturb_pair" if paired else "perturb"): {
+                "ms": per["perturb"], "launches": counts["perturb"], "GB/s": achieved, "frac_hbm": achieved / hbm},
             "restore": {"ms": per["restore"], "launches": counts["restore"],
                         "GB/s": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9,
                         "frac_hbm": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9 / hbm},
@@ -437,6 +450,10 @@ def main():
                                     "frac_alu": upd_ops / alu_peak,
                                     "ops_per_normal": alu_ops_per_normal, "normals_per_elem": n_normals_update},
             "shape": {"ms": per["shape"], "launches": counts["shape"]},
+            **({"perturb_partner": {"ms": per["partner"], "launches": counts["partner"],
+                                    "GB/s": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9,
+                                    "frac_hbm": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9 / hbm}}
+               if paired else {}),
         },
         "clocks": clk,
         "e2e": {"value": e2e, "unit": "params/s", "h2d_bytes_per_step": wl.K * wl.n_members * 4,
@@ -670,10 +687,13 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
 
     # each step's partition is built on a side stream while the previous step runs
     parts = es.ChunkPrefetcher(layout, K, lambda s: 1000 + s, chunk=chunk, tile_size=args.tile)
+    # random chunks spread every subspace over the arena: one partner buffer covers it
+    partner = None if args.no_partner else es.Partner(
+        torch.empty(layout.d_pad, dtype=arena.w.dtype, device="cuda"), 0)
 
     def step(s, events=None):
         subs = parts.take(s, events=events)
-        es.sync_step(arena, subs, s, cfg, d, rewards[s], joint=True, events=events)
+        es.sync_step(arena, subs, s, cfg, d, rewards[s], joint=True, events=events, partner=partner)
         if s + 1 < total:
             parts.prefetch(s + 1, events=events)
         return subs
@@ -710,7 +730,8 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
     # the update's roofline is the slower of its ALU and HBM bounds
     t_alu = 28.0 * P * mean_dk / (alu_peak * 1e12)
     t_hbm = 10.0 * mean_dk / (hbm * 1e9)
-    perturb_gbs = 6.0 * mean_dk / (per["perturb"] * 1e-3) / 1e9
+    paired = "partner" in per
+    perturb_gbs = (8.0 if paired else 6.0) * mean_dk / (per["perturb"] * 1e-3) / 1e9
     value = job_throughput(world, d, args.steps, ms * 1e-3)
     out = {
         "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
@@ -721,14 +742,17 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
                                "joint z-score, coefficient alpha/N_k",
                    "params": d, "K": K, "N": wl.n_members, "chunk": chunk, "sigma": wl.sigma, "alpha": wl.alpha,
                    "tile": args.tile, "l2": "inputs larger than L2, no flush"},
-        "roofline": {"bound": "hbm", "kernel": "perturb", "achieved": perturb_gbs, "peak": hbm, "unit": "GB/s",
-                     "frac": perturb_gbs / hbm, "traffic": None, "peak_source": "measured"},
+        "roofline": {"bound": "hbm", "kernel": "perturb_pair" if paired else "perturb", "achieved": perturb_gbs,
+                     "peak": hbm, "unit": "GB/s", "frac": perturb_gbs / hbm, "traffic": None,
+                     "peak_source": "measured"},
         "kernels": {
             "partition": {"ms": per["partition"], "launches": counts["partition"],
                           "note": "side-stream window, host tile building included; overlapped with "
                                   "the previous step"},
-            "perturb": {"ms": per["perturb"], "launches": counts["perturb"], "GB/s": perturb_gbs,
-                        "frac_hbm": perturb_gbs / hbm},
+            ("perturb_pair" if paired else "perturb"): {"ms": per["perturb"], "launches": counts["perturb"],
+                                                        "GB/s": perturb_gbs, "frac_hbm": perturb_gbs / hbm},
+            **({"perturb_partner": {"ms": per["partner"], "launches": counts["partner"],
+                                    "GB/s": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9}} if paired else {}),
             "restore": {"ms": per["restore"], "launches": counts["restore"],
                         "GB/s": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9},
             "update_fused_commit": {"ms": per["update"], "launches": counts["update"], "Tops": upd_tops,

@@ -306,6 +306,29 @@ int copes_hash_replay_mask(const copes_params *p, const copes_subspace *S, cudaS
 int copes_perturb(const copes_params *p, const copes_subspace *S, uint64_t seed,
                   float signed_sigma, cudaStream_t stream);
 
+/* Antithetic pair perturb (Eq. 8 for both members of one noise vector, no counterpart in
+ * the paper's implementation): one pass over S computes, for every g in S,
+ *   w[g]                          = round(fma( signed_sigma, eps_seed[g], theta[g]))
+ *   partner[g - partner_base]     = round(fma(-signed_sigma, eps_seed[g], theta[g]))
+ * i.e. w exactly as copes_perturb(signed_sigma) writes it, and the partner member's
+ * weights exactly as copes_perturb(-signed_sigma) would write them, from one generation
+ * of the noise.  partner: caller-owned device buffer of the working dtype (2 B per element
+ * for bf16, 4 B for fp32), 16-byte aligned, holding global indices
+ * [partner_base, partner_base + partner_len) at offsets 0 .. partner_len - 1; partner_base
+ * is a multiple of 4 and the range lies inside the arena (COPES_ERR_ALIGNMENT /
+ * COPES_ERR_SIZE otherwise).  An element of S outside that range is skipped and reported
+ * by copes_check (bit 16).  Entries of the buffer outside S are untouched. */
+int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t seed,
+                       float signed_sigma, void *partner, uint64_t partner_base,
+                       uint64_t partner_len, cudaStream_t stream);
+
+/* The partner member's perturb: w[g] = partner[g - partner_base] for g in S, a copy of
+ * the values copes_perturb_pair wrote.  Equal, bit for bit, to copes_perturb with the
+ * partner's signed sigma as long as theta is unchanged since that copes_perturb_pair.
+ * Reads neither theta nor the noise.  Buffer rules as for copes_perturb_pair. */
+int copes_perturb_partner(const copes_params *p, const copes_subspace *S, const void *partner,
+                          uint64_t partner_base, uint64_t partner_len, cudaStream_t stream);
+
 /* Restore (Sec. 3.3, Supp. A.8 "CPU Weight Backup", here an on-device fp32 master):
  *   w[g] = round(theta[g]) for g in S, bit-exact; outside S untouched. */
 int copes_restore(const copes_params *p, const copes_subspace *S, cudaStream_t stream);

@@ -9,7 +9,7 @@ from __future__ import annotations
 import ctypes
 import os
 from dataclasses import dataclass
-from typing import List, Optional, Sequence
+from typing import List, Optional, Sequence, Tuple
 
 import numpy as np
 import torch
@@ -92,6 +92,8 @@ SIGNATURES = {
     "copes_hash_replay_bytes": (_SZ, [_VP]),
     "copes_hash_replay_subspace": (_I32, [_VP, _I32, _U64, _I32, _VP, _SZ, _VP, _VP]),
     "copes_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
+    "copes_perturb_pair": (_I32, [_VP, _VP, _U64, _F32, _VP, _U64, _U64, _VP]),
+    "copes_perturb_partner": (_I32, [_VP, _VP, _VP, _U64, _U64, _VP]),
     "copes_restore": (_I32, [_VP, _VP, _VP]),
     "copes_context_commit": (_I32, [_VP, _VP, _VP]),
     "copes_shape_fitness": (_I32, [_VP, _I32, _VP, _I32, _VP, _VP]),
@@ -355,6 +357,58 @@ def hash_replay_partition(layout: Layout, K: int, seed: int, count: bool = True,
 def perturb(arena: Arena, sub: SubspaceHandle, seed: int, signed_sigma: float, stream=None) -> None:
     S = sub.struct()
     _check(load().copes_perturb(ctypes.byref(arena.params), ctypes.byref(S), seed, signed_sigma, _stream(stream)))
+
+
+def subspace_spans(arena: Arena, subs: Sequence[SubspaceHandle]) -> List[Tuple[int, int]]:
+    """[lo, hi) global-index span of each subspace (lo rounded down to a multiple of 4, as
+    partner buffers need), read from the device in one copy; (0, 0) for an empty one."""
+    spans = []
+    for sub in subs:
+        if sub.kind == SUBSPACE_TILES and sub.tensor.shape[0]:
+            spans.append(torch.stack([sub.tensor[:, 0].min(), sub.tensor[:, 1].max()]))
+        elif sub.kind == SUBSPACE_INDICES and sub.tensor.numel():
+            spans.append(torch.stack([sub.tensor[0], sub.tensor[-1] + 1]))
+        elif sub.kind == SUBSPACE_HASH_REPLAY:
+            spans.append(torch.tensor([0, arena.w.numel()], device=arena.w.device))
+        else:
+            spans.append(torch.zeros(2, dtype=torch.int64, device=arena.w.device))
+    if not spans:
+        return []
+    s = torch.stack(spans).cpu().numpy()
+    return [(int(lo) & ~3, int(hi)) if hi > lo else (0, 0) for lo, hi in s]
+
+
+def partner_buffer(arena: Arena, subs: Sequence[SubspaceHandle]) -> Tuple[torch.Tensor, int]:
+    """A partner buffer (working dtype) covering every element of `subs`, and its base
+    global index."""
+    spans = [x for x in subspace_spans(arena, subs) if x[1] > x[0]]
+    lo = min((x[0] for x in spans), default=0)
+    hi = max((x[1] for x in spans), default=0)
+    return torch.empty(max(hi - lo, 8), dtype=arena.w.dtype, device=arena.w.device), lo
+
+
+def _partner_view(arena: Arena, partner: torch.Tensor, base: int) -> torch.Tensor:
+    assert partner.is_cuda and partner.dtype == arena.w.dtype and partner.is_contiguous()
+    return partner[:max(0, min(partner.numel(), arena.w.numel() - base))]
+
+
+def perturb_pair(arena: Arena, sub: SubspaceHandle, seed: int, signed_sigma: float, partner: torch.Tensor,
+                 base: int = 0, stream=None) -> None:
+    """copes_perturb_pair: w as perturb(signed_sigma) and the partner member's weights
+    (-signed_sigma) into `partner` (element g at partner[g - base])."""
+    view = _partner_view(arena, partner, base)
+    S = sub.struct()
+    _check(load().copes_perturb_pair(ctypes.byref(arena.params), ctypes.byref(S), seed, signed_sigma,
+                                     _ptr(partner), base, view.numel(), _stream(stream)))
+
+
+def perturb_partner(arena: Arena, sub: SubspaceHandle, partner: torch.Tensor, base: int = 0,
+                    stream=None) -> None:
+    """copes_perturb_partner: w[g] = partner[g - base] for g in the subspace."""
+    view = _partner_view(arena, partner, base)
+    S = sub.struct()
+    _check(load().copes_perturb_partner(ctypes.byref(arena.params), ctypes.byref(S), _ptr(partner), base,
+                                        view.numel(), _stream(stream)))
 
 
 def restore(arena: Arena, sub: SubspaceHandle, stream=None) -> None:

@@ -164,12 +164,22 @@ void scaled_coeffs(float scale, copes::ScaledCoeffs &k) {
   for (int i = 0; i <= COPES_NORMAL_TAIL_DEGREE; ++i) k.tail[i] = scale * tail[i];
 }
 
+// The antithetic partner buffer (copes_perturb_pair / copes_perturb_partner).
+struct Partner {
+  const void *buf = nullptr;
+  uint64_t base = 0, len = 0;
+};
+
 int run_elementwise(int op, const copes_params *p, const copes_subspace *S, uint64_t seed,
-                    uint32_t tag, float a_val, float b_val, cudaStream_t s, const char *who) {
+                    uint32_t tag, float a_val, float b_val, cudaStream_t s, const char *who,
+                    const Partner &partner = Partner{}) {
   int rc = check_params(p, who);
   if (rc) return rc;
   if ((rc = check_subspace(S, who))) return rc;
   ElemArgs a = elem_args(p, S);
+  a.partner = const_cast<void *>(partner.buf);
+  a.partner_base = partner.base;
+  a.partner_len = partner.len;
   a.seed_lo = (uint32_t)seed;
   a.seed_hi = (uint32_t)(seed >> 32);
   a.tag = tag;
@@ -235,7 +245,8 @@ int copes_check(cudaStream_t stream) {
     return fail(COPES_ERR_DEVICE_CHECK,
                 "copes_check: a kernel's own check failed and it skipped the work (bits 0x%x: 1 = tile "
                 "outside the arena, 2 = gather index outside the arena, 4 = inconsistent partition "
-                "workspace or replay table, 8 = a bulk-copy wait ran out)",
+                "workspace or replay table, 8 = a bulk-copy wait ran out, 16 = an element outside "
+                "the partner buffer)",
                 bits);
   return COPES_OK;
 }
@@ -523,6 +534,38 @@ int copes_perturb(const copes_params *p, const copes_subspace *S, uint64_t seed,
   if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "copes_perturb: sigma is not finite");
   return run_elementwise(copes::kOpPerturb, p, S, seed, COPES_TAG_NOISE, signed_sigma, 0.0f, stream,
                          "copes_perturb");
+}
+
+static int check_partner(const copes_params *p, const void *buf, uint64_t base, uint64_t len,
+                         const char *who) {
+  if (!buf) return fail(COPES_ERR_INVALID_ARG, "%s: the partner buffer is NULL", who);
+  if (!aligned(buf, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: the partner buffer must be 16-byte aligned", who);
+  if (base % 4) return fail(COPES_ERR_ALIGNMENT, "%s: partner_base must be a multiple of 4", who);
+  if (p && (base > p->n_alloc || len > p->n_alloc - base))
+    return fail(COPES_ERR_SIZE, "%s: [partner_base, partner_base + partner_len) exceeds the arena", who);
+  return COPES_OK;
+}
+
+int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t seed,
+                       float signed_sigma, void *partner, uint64_t partner_base,
+                       uint64_t partner_len, cudaStream_t stream) {
+  const char *who = "copes_perturb_pair";
+  if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "%s: sigma is not finite", who);
+  int rc = check_params(p, who);
+  if (rc) return rc;
+  if ((rc = check_partner(p, partner, partner_base, partner_len, who))) return rc;
+  return run_elementwise(copes::kOpPerturbPair, p, S, seed, COPES_TAG_NOISE, signed_sigma, 0.0f, stream,
+                         who, Partner{partner, partner_base, partner_len});
+}
+
+int copes_perturb_partner(const copes_params *p, const copes_subspace *S, const void *partner,
+                          uint64_t partner_base, uint64_t partner_len, cudaStream_t stream) {
+  const char *who = "copes_perturb_partner";
+  int rc = check_params(p, who);
+  if (rc) return rc;
+  if ((rc = check_partner(p, partner, partner_base, partner_len, who))) return rc;
+  return run_elementwise(copes::kOpPartner, p, S, 0, 0, 0.0f, 0.0f, stream, who,
+                         Partner{partner, partner_base, partner_len});
 }
 
 int copes_restore(const copes_params *p, const copes_subspace *S, cudaStream_t stream) {

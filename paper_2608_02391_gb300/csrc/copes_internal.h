@@ -79,7 +79,8 @@ enum : unsigned {
   kErrTileRange = 1u,   // a tile outside [0, n_alloc) or longer than COPES_TILE_MAX
   kErrIndexRange = 2u,  // a gather index outside [0, n_alloc)
   kErrPartition = 4u,   // a partition kernel met an inconsistent workspace
-  kErrStageTimeout = 8u // a bulk-copy wait ran past its iteration limit
+  kErrStageTimeout = 8u, // a bulk-copy wait ran past its iteration limit
+  kErrPartnerRange = 16u // an element outside the partner buffer's range
 };
 
 // ---------------------------------------------------------------- launch arguments
@@ -105,10 +106,24 @@ struct ElemArgs {
   ScaledCoeffs coeffs;  // a * R's coefficients (perturb, init)
   uint32_t rk[20];      // Philox round keys of (seed_lo, seed_hi)
   float *gathered;      // INDICES: theta in list order instead of master[index[p]] (or NULL)
+  // kOpPerturbPair / kOpPartner: the antithetic partner's weights (working dtype), element
+  // g at partner[g - partner_base] for partner_base <= g < partner_base + partner_len
+  void *partner;
+  uint64_t partner_base, partner_len;
 };
 
 // kOpGather / kOpScatter copy theta between master and the gathered copy (INDICES only).
-enum ElemOp { kOpPerturb = 0, kOpRestore = 1, kOpInit = 2, kOpGather = 3, kOpScatter = 4 };
+// kOpPerturbPair writes w = rn(theta + a eps) and the partner member's rn(theta - a eps)
+// to the partner buffer; kOpPartner copies the partner buffer into w.
+enum ElemOp {
+  kOpPerturb = 0,
+  kOpRestore = 1,
+  kOpInit = 2,
+  kOpGather = 3,
+  kOpScatter = 4,
+  kOpPerturbPair = 5,
+  kOpPartner = 6
+};
 
 struct UpdateArgs {
   void *w;

@@ -1,6 +1,6 @@
 // Device pieces shared by the ES kernels of the tile / gather path (es_kernels.cu) and of
-// the partition-replay path (replay_kernels.cu): working-weight stores, the scaled normal
-// of one Philox word, and the update's prologue.
+// the partition-replay path (replay_kernels.cu): working-weight stores and the update's
+// prologue.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -35,13 +35,6 @@ struct WStore<float> {
     reinterpret_cast<float *>(w)[g] = v;
   }
 };
-
-// scale * eps + b for one word, with scale folded into the coefficients: one fma.
-__device__ __forceinline__ float scaled_normal_plus(uint32_t w, const ScaledCoeffs &k, float b) {
-  float x, r;
-  normal_parts(w, k.central, k.tail, x, r);
-  return __fmaf_rn(r, x, b);
-}
 
 // The update's prologue: folds the members into one weight per noise vector,
 //   w_j = sum_{i : noise(i) = j} sign_i f_i  (member order, fp32),

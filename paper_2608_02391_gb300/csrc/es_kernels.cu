@@ -31,11 +31,13 @@ __device__ __forceinline__ float index_noise(uint64_t g, uint32_t tag, uint32_t 
 template <int OP>
 constexpr uint32_t op_tag() { return OP == kOpInit ? COPES_TAG_INIT : COPES_TAG_NOISE; }
 
-// perturb: v = theta + a eps;  init: v = b + a eps;  restore: v = theta.  (q_lo, q_hi) is
-// the group's Philox counter g4 >> 2.
+// perturb: v = theta + a eps;  init: v = b + a eps;  restore: v = theta;  perturb pair:
+// v = theta + a eps and the partner's vp = theta - a eps.  (q_lo, q_hi) is the group's
+// Philox counter g4 >> 2.  Coefficients scaled by -a are the exact negatives of those
+// scaled by a, so vp equals, bit for bit, what kOpPerturb computes with scale -a.
 template <int OP>
 __device__ __forceinline__ void elem_values(const ElemArgs &a, uint32_t q_lo, uint32_t q_hi,
-                                            const float th[4], float v[4]) {
+                                            const float th[4], float v[4], float vp[4]) {
   if (OP == kOpRestore) {
 #pragma unroll
     for (int e = 0; e < 4; ++e) v[e] = th[e];
@@ -45,7 +47,11 @@ __device__ __forceinline__ void elem_values(const ElemArgs &a, uint32_t q_lo, ui
     float x[4], r[4];
     normal_parts4_x2(w, a.coeffs.central2, a.coeffs.tail, x, r);  // r = a * R(L)
 #pragma unroll
-    for (int e = 0; e < 4; ++e) v[e] = __fmaf_rn(r[e], x[e], OP == kOpPerturb ? th[e] : a.b);
+    for (int e = 0; e < 4; ++e) v[e] = __fmaf_rn(r[e], x[e], OP == kOpInit ? a.b : th[e]);
+    if (OP == kOpPerturbPair) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) vp[e] = __fmaf_rn(-r[e], x[e], th[e]);
+    }
   }
 }
 
@@ -76,15 +82,16 @@ __device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b,
     for (int i = 0; i < G; ++i) {
       const uint32_t o = off + 4u * kThreads * i;
       if (o >= len) continue;
-      float v[4];
+      float v[4], vp[4];
       if (HI0) {
-        elem_values<OP>(a, q0_lo + (o >> 2), 0u, th[i], v);
+        elem_values<OP>(a, q0_lo + (o >> 2), 0u, th[i], v, vp);
       } else {
         const uint64_t q = q0 + (o >> 2);
-        elem_values<OP>(a, (uint32_t)q, (uint32_t)(q >> 32), th[i], v);
+        elem_values<OP>(a, (uint32_t)q, (uint32_t)(q >> 32), th[i], v, vp);
       }
       if (OP == kOpInit) st_stream_f4(mt + o, make_float4(v[0], v[1], v[2], v[3]));
       WStore<WT>::full(a.w, b + o, v);
+      if (OP == kOpPerturbPair) WStore<WT>::full(a.partner, b + o - a.partner_base, vp);
     }
   }
 }
@@ -119,11 +126,12 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
     for (int i = 0; i < G; ++i) {
       const uint64_t g4 = base + 4ull * kThreads * i;
       if (g4 >= e) continue;
-      float v[4];
-      elem_values<OP>(a, (uint32_t)(g4 >> 2), (uint32_t)(g4 >> 34), th[i], v);
+      float v[4], vp[4];
+      elem_values<OP>(a, (uint32_t)(g4 >> 2), (uint32_t)(g4 >> 34), th[i], v, vp);
       if (full[i]) {
         if (OP == kOpInit) st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
         WStore<WT>::full(a.w, g4, v);
+        if (OP == kOpPerturbPair) WStore<WT>::full(a.partner, g4 - a.partner_base, vp);
       } else {
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -131,6 +139,7 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
           if (g >= b && g < e) {
             if (OP == kOpInit) master[g] = v[k];
             WStore<WT>::one(a.w, g, v[k]);
+            if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, g - a.partner_base, vp[k]);
           }
         }
       }
@@ -142,6 +151,11 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
 // thread for G = 8 groups in flight (measured 2% faster than G = 4 at 4 blocks, the next best).
 constexpr int kElemBlocksPerSM = 3;
 
+// A tile outside [partner_base, partner_base + partner_len) is skipped and flagged.
+__device__ __forceinline__ bool partner_covers(const ElemArgs &a, uint64_t b, uint64_t e) {
+  return b >= a.partner_base && e - a.partner_base <= a.partner_len;
+}
+
 template <int OP, typename WT, int G>
 __global__ void __launch_bounds__(kThreads, kElemBlocksPerSM) elem_tiles_kernel(const ElemArgs a) {
   const uint64_t t = blockIdx.x;
@@ -150,11 +164,63 @@ __global__ void __launch_bounds__(kThreads, kElemBlocksPerSM) elem_tiles_kernel(
     if (threadIdx.x == 0) flag_error(kErrTileRange);
     return;
   }
+  if (OP == kOpPerturbPair && !partner_covers(a, b, e)) {
+    if (threadIdx.x == 0) flag_error(kErrPartnerRange);
+    return;
+  }
   if (((b | e) & 3ull) == 0) {
     if ((e >> 34) == 0) elem_tile_aligned<OP, WT, G, true>(a, b, (uint32_t)(e - b));
     else elem_tile_aligned<OP, WT, G, false>(a, b, (uint32_t)(e - b));
   } else {
     elem_tile_ragged<OP, WT, G>(a, b, e);
+  }
+}
+
+// The partner member's perturb over TILES: w[g] = partner[g - partner_base], a copy of
+// the working dtype's bits (the values kOpPerturbPair wrote).  Aligned tiles move one
+// 4-element group (8 B bf16, 16 B fp32) per load; ragged tiles go element by element.
+template <typename WT>
+struct Group4;
+template <>
+struct Group4<__nv_bfloat16> {
+  using T = uint2;
+};
+template <>
+struct Group4<float> {
+  using T = uint4;
+};
+
+template <typename WT, int G>
+__global__ void __launch_bounds__(kThreads) partner_tiles_kernel(const ElemArgs a) {
+  const uint64_t t = blockIdx.x;
+  const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
+  if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
+    if (threadIdx.x == 0) flag_error(kErrTileRange);
+    return;
+  }
+  if (!partner_covers(a, b, e)) {
+    if (threadIdx.x == 0) flag_error(kErrPartnerRange);
+    return;
+  }
+  const WT *__restrict__ src = reinterpret_cast<const WT *>(a.partner) + (b - a.partner_base);
+  WT *__restrict__ dst = reinterpret_cast<WT *>(a.w) + b;
+  const uint32_t len = (uint32_t)(e - b);
+  if (((b | e) & 3ull) == 0) {  // partner_base is a multiple of 4, so src is aligned too
+    using V = typename Group4<WT>::T;
+    const V *__restrict__ vs = reinterpret_cast<const V *>(src);
+    V *__restrict__ vd = reinterpret_cast<V *>(dst);
+    const uint32_t n = len / 4;
+    for (uint32_t i0 = threadIdx.x; i0 < n; i0 += kThreads * G) {
+      V v[G];
+#pragma unroll
+      for (int k = 0; k < G; ++k)
+        if (i0 + kThreads * k < n) v[k] = __ldcs(vs + i0 + kThreads * k);
+#pragma unroll
+      for (int k = 0; k < G; ++k)
+        if (i0 + kThreads * k < n) __stcs(vd + i0 + kThreads * k, v[k]);
+    }
+  } else {
+    for (uint32_t i = threadIdx.x; i < len; i += kThreads) dst[i] = src[i];
   }
 }
 
@@ -186,8 +252,14 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
         flag_error(kErrIndexRange);
         ok[u] = false;
       }
+      if ((OP == kOpPerturbPair || OP == kOpPartner) && ok[u] &&
+          ((uint64_t)g[u] < a.partner_base || (uint64_t)g[u] - a.partner_base >= a.partner_len)) {
+        flag_error(kErrPartnerRange);
+        ok[u] = false;
+      }
       const bool from_gathered = GATH && OP != kOpGather;
-      th[u] = (OP != kOpInit && ok[u]) ? (from_gathered ? gath[first + p] : master[g[u]]) : 0.0f;
+      const bool reads_theta = OP != kOpInit && OP != kOpPartner;
+      th[u] = (reads_theta && ok[u]) ? (from_gathered ? gath[first + p] : master[g[u]]) : 0.0f;
     }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
@@ -198,8 +270,12 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
       } else if constexpr (OP == kOpScatter) {
         master[g[u]] = th[u];
         continue;
+      } else if constexpr (OP == kOpPartner) {
+        const uint64_t gi = (uint64_t)g[u];
+        reinterpret_cast<WT *>(a.w)[gi] = reinterpret_cast<const WT *>(a.partner)[gi - a.partner_base];
+        continue;
       } else {
-        float v;
+        float v, vp = 0.0f;
         if (OP == kOpRestore) {
           v = th[u];
         } else {
@@ -208,13 +284,17 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
           philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, op_tag<OP>(), a.rk, x);
           const uint32_t sel = (uint32_t)g[u] & 3u;
           const uint32_t wd = sel == 0 ? x[0] : (sel == 1 ? x[1] : (sel == 2 ? x[2] : x[3]));
-          v = scaled_normal_plus(wd, a.coeffs, OP == kOpPerturb ? th[u] : a.b);
+          float xv, r;
+          normal_parts(wd, a.coeffs.central, a.coeffs.tail, xv, r);  // r = a * R(L)
+          v = __fmaf_rn(r, xv, OP == kOpInit ? a.b : th[u]);
+          if (OP == kOpPerturbPair) vp = __fmaf_rn(-r, xv, th[u]);
         }
         if (OP == kOpInit) {
           if (GATH) gath[first + threadIdx.x + kThreads * u] = v;
           else master[g[u]] = v;
         }
         WStore<WT>::one(a.w, (uint64_t)g[u], v);
+        if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, (uint64_t)g[u] - a.partner_base, vp);
       }
     }
   });
@@ -230,7 +310,10 @@ static cudaError_t launch_elem_typed(int kind, const ElemArgs &a, cudaStream_t s
   } else if (kind == COPES_SUBSPACE_TILES) {
     if (a.n_tiles == 0) return cudaSuccess;
     constexpr int G = 8;
-    elem_tiles_kernel<OP, WT, G><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+    if constexpr (OP == kOpPartner)
+      partner_tiles_kernel<WT, G><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+    else
+      elem_tiles_kernel<OP, WT, G><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
   } else {
     if (a.n_index == 0) return cudaSuccess;
     const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
@@ -252,6 +335,8 @@ cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, c
     case kOpRestore: return launch_elem_op<kOpRestore>(kind, dtype, a, s);
     case kOpGather: return launch_elem_op<kOpGather>(kind, dtype, a, s);
     case kOpScatter: return launch_elem_op<kOpScatter>(kind, dtype, a, s);
+    case kOpPerturbPair: return launch_elem_op<kOpPerturbPair>(kind, dtype, a, s);
+    case kOpPartner: return launch_elem_op<kOpPartner>(kind, dtype, a, s);
     default: return launch_elem_op<kOpInit>(kind, dtype, a, s);
   }
 }

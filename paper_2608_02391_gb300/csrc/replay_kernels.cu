@@ -184,14 +184,27 @@ __global__ void __launch_bounds__(kThreads) replay_elem_kernel(const __grid_cons
   __syncthreads();
   float *__restrict__ master = a.master;
   replay_stream<BATCH, MASK>(r, a.n_alloc, s_buf[threadIdx.x >> 5], s_g0, s_pool, &s_pool_n,
-                             [&](const uint64_t (&g)[U], const bool (&ok)[U]) {
+                             [&](const uint64_t (&g)[U], const bool (&ok_in)[U]) {
+    bool ok[U];
     float th[U];
 #pragma unroll
-    for (int u = 0; u < U; ++u) th[u] = (OP != kOpInit && ok[u]) ? master[g[u]] : 0.0f;
+    for (int u = 0; u < U; ++u) {
+      ok[u] = ok_in[u];
+      if ((OP == kOpPerturbPair || OP == kOpPartner) && ok[u] &&
+          (g[u] < a.partner_base || g[u] - a.partner_base >= a.partner_len)) {
+        replay_flag(kErrPartnerRange);
+        ok[u] = false;
+      }
+      th[u] = (OP != kOpInit && OP != kOpPartner && ok[u]) ? master[g[u]] : 0.0f;
+    }
 #pragma unroll
     for (int u = 0; u < U; ++u) {
       if (!ok[u]) continue;
-      float v;
+      if constexpr (OP == kOpPartner) {
+        reinterpret_cast<WT *>(a.w)[g[u]] = reinterpret_cast<const WT *>(a.partner)[g[u] - a.partner_base];
+        continue;
+      }
+      float v, vp = 0.0f;
       if (OP == kOpRestore) {
         v = th[u];
       } else {
@@ -200,10 +213,14 @@ __global__ void __launch_bounds__(kThreads) replay_elem_kernel(const __grid_cons
         philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, replay_tag<OP>(), a.rk, x);
         const uint32_t sel = (uint32_t)g[u] & 3u;
         const uint32_t wd = sel == 0 ? x[0] : (sel == 1 ? x[1] : (sel == 2 ? x[2] : x[3]));
-        v = scaled_normal_plus(wd, a.coeffs, OP == kOpPerturb ? th[u] : a.b);
+        float xv, r;
+        normal_parts(wd, a.coeffs.central, a.coeffs.tail, xv, r);  // r = a * R(L)
+        v = __fmaf_rn(r, xv, OP == kOpInit ? a.b : th[u]);
+        if (OP == kOpPerturbPair) vp = __fmaf_rn(-r, xv, th[u]);
         if (OP == kOpInit) master[g[u]] = v;
       }
       WStore<WT>::one(a.w, g[u], v);
+      if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, g[u] - a.partner_base, vp);
     }
   }, [] {});
 }
@@ -318,6 +335,8 @@ static cudaError_t launch_replay_elem_dtype(int op, const ElemArgs &a, const Rep
   switch (op) {
     case kOpPerturb: return launch_replay_elem_typed<kOpPerturb, WT>(a, r, s);
     case kOpRestore: return launch_replay_elem_typed<kOpRestore, WT>(a, r, s);
+    case kOpPerturbPair: return launch_replay_elem_typed<kOpPerturbPair, WT>(a, r, s);
+    case kOpPartner: return launch_replay_elem_typed<kOpPartner, WT>(a, r, s);
     default: return launch_replay_elem_typed<kOpInit, WT>(a, r, s);
   }
 }

@@ -46,6 +46,53 @@ class ESConfig:
     base_seed: int = 33
 
 
+@dataclass
+class Partner:
+    """Buffer for the antithetic partner's weights (copes_perturb_pair): element g of the
+    arena at buf[g - base], in the working dtype.  Partner.covering(arena, subs) sizes one
+    for every element of `subs`."""
+    buf: torch.Tensor
+    base: int
+
+    @classmethod
+    def covering(cls, arena: copes.Arena, subs: Sequence[copes.SubspaceHandle]) -> "Partner":
+        """One buffer covering every element of `subs` (for steps that perturb them all,
+        e.g. sync_step)."""
+        buf, base = copes.partner_buffer(arena, subs)
+        return cls(buf, base)
+
+    @classmethod
+    def per_subspace(cls, arena: copes.Arena, subs: Sequence[copes.SubspaceHandle]) -> List["Partner"]:
+        """One buffer as wide as the widest subspace's span, shared by a Partner per
+        subspace with that subspace's own base (round-robin visits use one at a time)."""
+        spans = copes.subspace_spans(arena, subs)
+        width = max((hi - lo for lo, hi in spans), default=0)
+        buf = torch.empty(max(width, 8), dtype=arena.w.dtype, device=arena.w.device)
+        return [cls(buf, lo) for lo, _ in spans]
+
+
+def perturb_members(arena: copes.Arena, sub: copes.SubspaceHandle, members: Sequence[int], nid, sign,
+                    seeds, s_k: float, live: Callable[[int], None], partner: Optional[Partner] = None,
+                    events: Optional[dict] = None) -> None:
+    """Perturbs each member of `members` in order (Eq. 8) and calls live(i) while member i's
+    perturbation is in place.  With a partner buffer, a member whose successor shares its
+    noise vector with the opposite sign (an antithetic pair) is perturbed by
+    copes_perturb_pair, and the successor's weights are then copied in from the buffer:
+    one noise generation per pair, bit-identical weights."""
+    staged = None  # the member whose weights the partner buffer holds
+    for pos, i in enumerate(members):
+        nxt = members[pos + 1] if pos + 1 < len(members) else None
+        seed, ss = int(seeds[nid[i]]), float(sign[i]) * s_k
+        if staged == i:
+            _timed(events, "partner", lambda: copes.perturb_partner(arena, sub, partner.buf, partner.base))
+        elif partner is not None and nxt is not None and nid[nxt] == nid[i] and sign[nxt] == -sign[i]:
+            _timed(events, "perturb", lambda: copes.perturb_pair(arena, sub, seed, ss, partner.buf, partner.base))
+            staged = nxt
+        else:
+            _timed(events, "perturb", lambda: copes.perturb(arena, sub, seed, ss))
+        live(i)
+
+
 def sigma_k(cfg: ESConfig, d: int, d_k: int) -> float:
     """Eq. 11 when dimension-aware, else the configured sigma."""
     return copes.sigma_eff(cfg.sigma, d, d_k, cfg.dimension_aware)
@@ -55,17 +102,16 @@ def round_robin_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, ite
                       cfg: ESConfig, d: int, rewards: torch.Tensor,
                       evaluate: Optional[Callable[[int], None]] = None,
                       fitness_out: Optional[torch.Tensor] = None,
-                      events: Optional[dict] = None) -> torch.Tensor:
+                      events: Optional[dict] = None, partner: Optional[Partner] = None) -> torch.Tensor:
     """One ES iteration on subspace k.  `rewards` (device fp32 [N]) holds the members'
     rewards; `evaluate(i)` runs while member i's perturbation is live (it may write
-    rewards[i]).  Returns the shaped fitness."""
+    rewards[i]).  `partner`: perturb antithetic pairs with one noise generation
+    (perturb_members).  Returns the shaped fitness."""
     nid, sign, P = copes.member_table(cfg.n_members, cfg.pairing)
     seeds = copes.member_seeds(cfg.base_seed, iteration, k, P)
     s_k = sigma_k(cfg, d, sub.numel)
-    for i in range(cfg.n_members):
-        _timed(events, "perturb", lambda: copes.perturb(arena, sub, int(seeds[nid[i]]), float(sign[i]) * s_k))
-        if evaluate is not None:
-            evaluate(i)
+    perturb_members(arena, sub, range(cfg.n_members), nid, sign, seeds, s_k,
+                    evaluate if evaluate is not None else (lambda i: None), partner, events)
     _timed(events, "restore", lambda: copes.restore(arena, sub))
     f = fitness_out if fitness_out is not None else torch.empty_like(rewards)
     _timed(events, "shape", lambda: copes.shape_fitness(rewards, cfg.shaping, out=f))
@@ -102,10 +148,12 @@ def backup_visit(arena: copes.BackupArena, sub: copes.SubspaceHandle, k: int, it
 def sync_step(arena: copes.Arena, subs: Sequence[copes.SubspaceHandle], iteration: int,
               cfg: ESConfig, d: int, rewards: torch.Tensor,
               evaluate: Optional[Callable[[int, int], None]] = None,
-              joint: bool = True, events: Optional[dict] = None) -> torch.Tensor:
+              joint: bool = True, events: Optional[dict] = None,
+              partner: Optional[Partner] = None) -> torch.Tensor:
     """Algorithm 1: N = cfg.n_members split into N_k = N / K per subspace; rewards is the
     device fp32 [N] vector laid out subspace by subspace (member i of subspace k at
-    k N_k + i).  evaluate(k, i) runs while that member's perturbation is live."""
+    k N_k + i).  evaluate(k, i) runs while that member's perturbation is live.  `partner`
+    (covering every subspace): antithetic pairs with one noise generation."""
     K = len(subs)
     if cfg.n_members % K:
         raise ValueError("N must be divisible by K (Sec. 3.2)")
@@ -114,11 +162,9 @@ def sync_step(arena: copes.Arena, subs: Sequence[copes.SubspaceHandle], iteratio
     seeds = [copes.member_seeds(cfg.base_seed, iteration, k, P) for k in range(K)]
     for k, sub in enumerate(subs):
         s_k = sigma_k(cfg, d, sub.numel)
-        for i in range(n_k):
-            _timed(events, "perturb",
-                   lambda: copes.perturb(arena, sub, int(seeds[k][nid[i]]), float(sign[i]) * s_k))
-            if evaluate is not None:
-                evaluate(k, i)
+        perturb_members(arena, sub, range(n_k), nid, sign, seeds[k], s_k,
+                        (lambda i: evaluate(k, i)) if evaluate is not None else (lambda i: None),
+                        partner, events)
         # the next subspace is evaluated under the same context
         _timed(events, "restore", lambda: copes.restore(arena, sub))
     if joint:
@@ -239,7 +285,8 @@ def gather_rewards(local: np.ndarray, n_members: int, group=None) -> np.ndarray:
 
 def population_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iteration: int,
                      cfg: ESConfig, d: int, evaluate: Callable[[int], float], group=None,
-                     fitness_out: Optional[torch.Tensor] = None) -> torch.Tensor:
+                     fitness_out: Optional[torch.Tensor] = None,
+                     partner: Optional[Partner] = None) -> torch.Tensor:
     """One ES iteration on subspace k, population-parallel over the ranks of `group`.
     Every rank holds the same theta; rank r evaluates members member_slice(r, R, N):
     perturb, evaluate(i) -> reward (host float) while the perturbation is live, and
@@ -252,9 +299,11 @@ def population_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iter
     seeds = copes.member_seeds(cfg.base_seed, iteration, k, P)
     s_k = sigma_k(cfg, d, sub.numel)
     local = np.zeros(N, np.float32)
-    for i in member_slice(rank, world, N):
-        copes.perturb(arena, sub, int(seeds[nid[i]]), float(sign[i]) * s_k)
+
+    def live(i):
         local[i] = np.float32(evaluate(i))
+
+    perturb_members(arena, sub, member_slice(rank, world, N), nid, sign, seeds, s_k, live, partner)
     copes.restore(arena, sub)
     rewards = torch.from_numpy(gather_rewards(local, N, group)).to(arena.w.device)
     f = fitness_out if fitness_out is not None else torch.empty_like(rewards)

@@ -247,3 +247,27 @@ def test_replay_mask_arguments_are_rejected_before_any_launch(lib):
     assert lib.copes_hash_replay_mask(ctypes.byref(p), ctypes.byref(S), None) == copes.ERR_INVALID_ARG
     S.replay_mask = fake + 4
     assert lib.copes_hash_replay_mask(ctypes.byref(p), ctypes.byref(S), None) == copes.ERR_ALIGNMENT
+
+
+def test_partner_buffer_arguments_are_rejected_before_any_launch(lib):
+    """copes_perturb_pair / copes_perturb_partner: the partner buffer must be non-NULL,
+    16-byte aligned, start at a multiple of 4 and lie inside the arena."""
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    p = copes.Params(fake, fake, 1000, copes.BF16)
+    s = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
+    pair, partner = lib.copes_perturb_pair, lib.copes_perturb_partner
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, None, 0, 1000, None) == copes.ERR_INVALID_ARG
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake + 2, 0, 1000, None) == copes.ERR_ALIGNMENT
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake, 6, 900, None) == copes.ERR_ALIGNMENT
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake, 8, 993, None) == copes.ERR_SIZE
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake, 1004, 0, None) == copes.ERR_SIZE
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, float("inf"), fake, 0, 1000, None) == copes.ERR_INVALID_ARG
+    assert partner(ctypes.byref(p), ctypes.byref(s), None, 0, 1000, None) == copes.ERR_INVALID_ARG
+    assert partner(ctypes.byref(p), ctypes.byref(s), fake + 8, 0, 1000, None) == copes.ERR_ALIGNMENT
+    assert partner(ctypes.byref(p), ctypes.byref(s), fake, 2, 10, None) == copes.ERR_ALIGNMENT
+    assert partner(ctypes.byref(p), ctypes.byref(s), fake, 0, 1001, None) == copes.ERR_SIZE
+    bad = copes.Subspace(9, None, 0, None, 0)
+    assert partner(ctypes.byref(p), ctypes.byref(bad), fake, 0, 1000, None) == copes.ERR_INVALID_ARG
+    q = copes.Params(fake, fake + 4, 1000, copes.BF16)  # misaligned master
+    assert partner(ctypes.byref(q), ctypes.byref(s), fake, 0, 1000, None) == copes.ERR_ALIGNMENT

@@ -1,0 +1,199 @@
+"""Antithetic pair perturb (copes_perturb_pair / copes_perturb_partner) against the oracle
+and against two independent perturbs, for every subspace kind and both working dtypes:
+the member's weights, the partner's weights written to the buffer and then copied in, the
+buffer and the weights left untouched outside S, the buffer's range check, and whole ES
+visits and Algorithm 1 steps with and without the buffer."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from tolerances import assert_bf16_close, assert_perturb_fp32_close
+
+pytestmark = pytest.mark.gpu
+
+N_ALLOC = 60_000
+RANGES = [(3, 9_001), (9_001, 9_003), (12_345, 30_000), (30_064, 30_065), (40_001, 59_997)]
+
+
+@pytest.fixture(scope="module")
+def copes():
+    from paper_2608_02391_gb300 import copes as c
+    c.load()
+    return c
+
+
+def theta_np(n=N_ALLOC, seed=0):
+    return (np.random.default_rng(seed).standard_normal(n) * 0.02).astype(np.float32)
+
+
+def canary(n, dtype, seed):
+    rng = np.random.default_rng(seed)
+    if dtype == torch.bfloat16:
+        b = (rng.standard_normal(n).astype(np.float32) * 0.05).view(np.uint32) >> 16
+        return torch.from_numpy(b.astype(np.int16)).view(torch.bfloat16).cuda()
+    return torch.from_numpy((rng.standard_normal(n) * 0.05).astype(np.float32)).cuda()
+
+
+def bits(t):
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).cpu().numpy().view(np.uint16)
+    return t.cpu().numpy().view(np.uint32)
+
+
+def mask_of(ranges, n=N_ALLOC):
+    m = np.zeros(n, bool)
+    for b, e in ranges:
+        m[b:e] = True
+    return m
+
+
+def make_sub(copes, kind, ranges, arena):
+    if kind.startswith("tiles"):
+        return copes.tiles_from_ranges(ranges, tile_size=int(kind.split(":")[1]))
+    idx = np.concatenate([np.arange(b, e) for b, e in ranges]).astype(np.int64)
+    sub = copes.SubspaceHandle(copes.SUBSPACE_INDICES, torch.from_numpy(idx).cuda(), idx.size)
+    if kind == "gathered":
+        sub.gathered = torch.empty(idx.size, dtype=torch.float32, device="cuda")
+        copes.gather_master(arena, sub)
+    return sub
+
+
+def check_member(got_bits, dtype, g, theta_in, seed, ss):
+    """The bits of one member's weights at g against the oracle's perturb."""
+    if dtype == torch.bfloat16:
+        ref_bits, _ = oracle.perturb_at(g, theta_in, seed, ss, oracle.BF16)
+        scale = np.maximum(np.abs(theta_in), np.abs(np.float32(ss) * oracle.noise(seed, g)))
+        assert_bf16_close(got_bits, ref_bits.astype(np.uint16), scale)
+    else:
+        _, exact = oracle.perturb_at(g, theta_in, seed, ss, oracle.FP32)
+        assert_perturb_fp32_close(got_bits.view(np.float32), exact, theta_in,
+                                  np.float32(ss) * oracle.noise(seed, g))
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("kind", ["tiles:4096", "tiles:1000", "indices", "gathered"])
+@pytest.mark.parametrize("ranges,base", [(RANGES, 0), (RANGES[2:], 12_344)])
+def test_pair_equals_two_perturbs_and_the_oracle(copes, dtype, kind, ranges, base):
+    theta = theta_np()
+    inside = mask_of(ranges)
+    g = np.nonzero(inside)[0].astype(np.uint64)
+    w0 = canary(N_ALLOC, dtype, 9)
+    ref = copes.Arena(w0.clone(), torch.from_numpy(theta.copy()).cuda())
+    arena = copes.Arena(w0.clone(), torch.from_numpy(theta.copy()).cuda())
+    sub_ref, sub = make_sub(copes, kind, ranges, ref), make_sub(copes, kind, ranges, arena)
+    buf = canary(N_ALLOC - base, dtype, 5)
+    buf0 = bits(buf).copy()
+    for seed, ss in [(11, 2e-3), (2**40 + 5, -1e-3)]:
+        copes.perturb(ref, sub_ref, seed, ss)
+        plus = bits(ref.w).copy()
+        copes.perturb(ref, sub_ref, seed, -ss)
+        minus = bits(ref.w).copy()
+        copes.perturb_pair(arena, sub, seed, ss, buf, base)
+        got = bits(arena.w)
+        assert np.array_equal(got, plus)  # w exactly as copes_perturb(+ss), untouched outside S
+        pb = bits(buf)
+        assert np.array_equal(pb[g.astype(np.int64) - base], minus[inside])
+        assert np.array_equal(pb[~inside[base:]], buf0[~inside[base:]])  # the buffer outside S
+        check_member(pb[g.astype(np.int64) - base], dtype, g, theta[inside], seed, -ss)
+        check_member(got[inside], dtype, g, theta[inside], seed, ss)
+        copes.perturb_partner(arena, sub, buf, base)
+        assert np.array_equal(bits(arena.w), minus)
+    copes.check()
+
+
+@pytest.mark.parametrize("masked", [False, True])
+def test_pair_on_replayed_hash_subspaces(copes, masked):
+    layout = copes.Layout([20_000, 7, 39_000])
+    n = layout.d_pad
+    theta = theta_np(n)
+    w0 = canary(n, torch.bfloat16, 9)
+    ref = copes.Arena(w0.clone(), torch.from_numpy(theta.copy()).cuda())
+    arena = copes.Arena(w0.clone(), torch.from_numpy(theta.copy()).cuda())
+    for k, sub in enumerate(copes.hash_replay_partition(layout, 4, 77)):
+        if masked:
+            copes.hash_replay_mask(arena, sub)
+        buf = canary(n, torch.bfloat16, 5 + k)
+        copes.perturb(ref, sub, 3 + k, 1e-3)
+        plus = bits(ref.w).copy()
+        copes.perturb(ref, sub, 3 + k, -1e-3)
+        minus = bits(ref.w).copy()
+        copes.perturb_pair(arena, sub, 3 + k, 1e-3, buf, 0)
+        assert np.array_equal(bits(arena.w), plus)
+        copes.perturb_partner(arena, sub, buf, 0)
+        assert np.array_equal(bits(arena.w), minus)
+    copes.check()
+
+
+@pytest.mark.parametrize("kind", ["tiles:4096", "indices"])
+def test_partner_range_is_checked_without_faulting(copes, kind):
+    """A buffer range that misses part of S: the kernels skip the missing elements (whole
+    tiles for TILES), write nothing past the range, and copes_check reports bit 16."""
+    theta = theta_np()
+    arena = copes.Arena(canary(N_ALLOC, torch.bfloat16, 9), torch.from_numpy(theta.copy()).cuda())
+    sub = make_sub(copes, kind, RANGES, arena)
+    big = canary(N_ALLOC, torch.bfloat16, 5)
+    before = bits(big).copy()
+    short = 20_000  # the range [0, 20000) misses the subspace's upper elements
+    copes.perturb_pair(arena, sub, 1, 1e-3, big[:short], 0)
+    with pytest.raises(copes.CopesError) as e:
+        copes.check()
+    assert e.value.code == copes.ERR_DEVICE_CHECK and "bits 0x10" in str(e.value)
+    assert np.array_equal(bits(big)[short:], before[short:])
+    copes.perturb_partner(arena, sub, big[:short], 0)
+    with pytest.raises(copes.CopesError):
+        copes.check()
+    copes.check()  # cleared
+
+
+def visit_trace(copes, es, partner_on, kind):
+    n = 1 << 18
+    theta = theta_np(n, 3)
+    arena = copes.Arena(torch.from_numpy(theta.copy()).cuda().to(torch.bfloat16),
+                        torch.from_numpy(theta.copy()).cuda())
+    layout = copes.Layout([n // 2, n // 2 - 100])
+    subs = (es.build_subspaces(layout, "contiguous", 3, tile_size=4096) if kind == "tiles"
+            else copes.hash_partition(layout, 3, 5))
+    partner = es.Partner.covering(arena, subs) if partner_on else None
+    cfg = es.ESConfig(n_members=8, sigma=1e-3, alpha=5e-4)
+    rng = np.random.default_rng(1)
+    trace = []
+    for k, sub in enumerate(subs):
+        r = torch.from_numpy(rng.standard_normal(8).astype(np.float32)).cuda()
+
+        def ev(i):  # what a rollout would see: the live weights' bits
+            trace.append(int(arena.w.view(torch.int16).to(torch.int64).mul(i + 1).sum()))
+
+        es.round_robin_visit(arena, sub, k, 0, cfg, n, r, evaluate=ev, partner=partner)
+    copes.check()
+    return trace, bits(arena.w), arena.master.cpu().numpy()
+
+
+@pytest.mark.parametrize("kind", ["tiles", "indices"])
+def test_visit_with_partner_buffer_is_bit_identical(copes, kind):
+    from paper_2608_02391_gb300 import es
+    t0, w0, m0 = visit_trace(copes, es, False, kind)
+    t1, w1, m1 = visit_trace(copes, es, True, kind)
+    assert t0 == t1 and len(t0) == 24
+    assert np.array_equal(w0, w1)
+    assert np.array_equal(m0.view(np.uint32), m1.view(np.uint32))
+
+
+def test_sync_step_with_partner_buffer_is_bit_identical(copes):
+    from paper_2608_02391_gb300 import es
+    n, K, N, chunk = 1 << 18, 4, 16, 4096
+    layout = copes.Layout([n])
+    cfg = es.ESConfig(n_members=N, sigma=1e-3, alpha=5e-4, convention=copes.COEF_PAPER, dimension_aware=True)
+    rewards = torch.from_numpy(np.random.default_rng(4).standard_normal(N).astype(np.float32)).cuda()
+    out = []
+    for use in (False, True):
+        theta = theta_np(n, 8)
+        arena = copes.Arena(torch.from_numpy(theta.copy()).cuda().to(torch.bfloat16),
+                            torch.from_numpy(theta.copy()).cuda())
+        subs = es.build_subspaces(layout, "random_chunks", K, seed=9, chunk=chunk)
+        partner = es.Partner.covering(arena, subs) if use else None
+        for step in range(2):
+            es.sync_step(arena, subs, step, cfg, n, rewards, partner=partner)
+        out.append((bits(arena.w), arena.master.cpu().numpy().view(np.uint32)))
+    copes.check()
+    assert np.array_equal(out[0][0], out[1][0]) and np.array_equal(out[0][1], out[1][1])
