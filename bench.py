@@ -53,13 +53,20 @@ METRIC = "ES-iteration params/s and HBM GB/s at 4B bf16 (N=32), % of roofline on
 FALLBACK_HBM_GBS = 6800.0
 
 # ncu DRAM bytes per element of the dominant kernel (the pair perturb, or the plain perturb
-# under --no-partner; bf16) from one capture each; a figure is dropped (traffic = null)
+# under --weights single; bf16) from one capture each; a figure is dropped (traffic = null)
 # when es_kernels.cu or copes_device.cuh no longer matches the hash it was taken on.
 NCU_TRAFFIC = {
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "6645acd4b5b44240",
-                     "bytes_per_elem": 7.231, "capture": "profiles/perturb_pair_4b_slice.md"},
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "e307f929a5d1d206",
+                     "bytes_per_elem": 7.228, "capture": "profiles/perturb_pair_4b_slice.md"},
     "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "fd276ea14451ff07",
                 "bytes_per_elem": 5.414, "capture": "profiles/perturb_4b_slice.md"},
+}
+
+
+WEIGHTS_MODES = {
+    "dual": "two bf16 copies: antithetic member 2j evaluated on w, 2j+1 on w2, both written by one pair perturb",
+    "partner": "one bf16 copy: member 2j+1 copied in from the pair perturb's partner buffer",
+    "single": "one bf16 copy: every member perturbed from theta",
 }
 
 
@@ -73,8 +80,10 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
-    ap.add_argument("--no-partner", action="store_true",
-                    help="perturb every member from theta (no antithetic partner buffer)")
+    ap.add_argument("--weights", default="dual", choices=["dual", "partner", "single"],
+                    help="dual: two working-weight copies, antithetic members 2j on w and 2j+1 on w2 "
+                         "(one pair perturb per pair); partner: one copy, member 2j+1 copied in from a "
+                         "partner buffer; single: one copy, every member perturbed from theta")
     ap.add_argument("--cpu-cores", type=int, default=0,
                     help="processes of the oracle's CPU sample (0: every core this process may use)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -286,13 +295,14 @@ def workload_config(wl, args):
     return {"workload": "4B decoder-shaped bf16 set, fp32 master, K=8 layer blocks, N=32 antithetic",
             "params": wl.d, "layers": 36, "hidden": 2560, "mlp": 9728, "vocab": 151936, "tied": True,
             "K": wl.K, "N": wl.n_members, "sigma": wl.sigma, "alpha": wl.alpha, "shaping": wl.shaping,
-            "tile": args.tile, "l2": "inputs larger than L2 (24 GB resident per step), no flush"}
+            "tile": args.tile, "working_weights": WEIGHTS_MODES[args.weights],
+            "l2": "inputs larger than L2 (24 GB or more resident per step), no flush"}
 
 
 # -------------------------------------------------------------------------- GPU leg
-def make_arena(copes, torch, wl, layout):
+def make_arena(copes, torch, wl, layout, dual=False):
     """Seeded synthetic weights: fp32 master ~ N(0, init_scale^2), norm tensors 1.0, and
-    w = bf16(master)."""
+    w = bf16(master) (and w2 = w for two working copies)."""
     master = torch.empty(layout.d_pad, dtype=torch.float32, device="cuda")
     gen = torch.Generator(device="cuda")
     gen.manual_seed(wl.init_seed)
@@ -301,7 +311,8 @@ def make_arena(copes, torch, wl, layout):
     for t, ten in enumerate(wl.tensors):
         if ten.kind == "norm":
             master[int(offs[t]):int(offs[t]) + ten.numel].fill_(1.0)
-    return copes.Arena(master.to(torch.bfloat16), master)
+    w = master.to(torch.bfloat16)
+    return copes.Arena(w, master, w2=w.clone() if dual else None)
 
 
 def main():
@@ -328,7 +339,7 @@ def main():
 
     layout = copes.Layout(wl.numel)
     d = wl.d
-    arena = make_arena(copes, torch, wl, layout)
+    arena = make_arena(copes, torch, wl, layout, dual=args.weights == "dual")
     cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping=wl.shaping)
     total_steps = args.warmup + args.steps + args.e2e_steps
     rewards_host = workloads.reward_stream(wl, total_steps * wl.K)  # [steps*K, N]
@@ -339,7 +350,12 @@ def main():
     tile_buf = [s.tensor for s in subs]
     # antithetic pairs: one noise generation per pair, the partner's weights staged in a
     # buffer as wide as the widest subspace
-    partners = [None] * wl.K if args.no_partner else es.Partner.per_subspace(arena, subs)
+    if args.weights == "dual":
+        partners = [es.Partner.second_copy(arena)] * wl.K
+    elif args.weights == "partner":
+        partners = es.Partner.per_subspace(arena, subs)
+    else:
+        partners = [None] * wl.K
 
     import ctypes
     L = copes.load()
@@ -409,10 +425,14 @@ def main():
     mean_dk = float(np.mean(d_k))
     peaks, peak_src = measured_peaks()
     hbm = float(peaks["hbm_gbs"])
-    paired = "partner" in per
+    paired = args.weights != "single"
+    dual = args.weights == "dual"
     # the pair perturb reads theta (4 B) and writes w and the partner's weights (2 + 2 B);
-    # the partner copy reads and writes 2 B; a plain perturb reads 4 B and writes 2 B
+    # the partner copy reads and writes 2 B; a plain perturb reads 4 B and writes 2 B.
+    # With two working copies, restore and the fused commit write both (+2 B each).
     perturb_bytes = (8.0 if paired else 6.0) * mean_dk
+    restore_bytes = (8.0 if dual else 6.0) * mean_dk
+    update_bytes = (12.0 if dual else 10.0) * mean_dk
     achieved = perturb_bytes / (per["perturb"] * 1e-3) / 1e9
     ncu = NCU_TRAFFIC["perturb_pair" if paired else "perturb"]
     traffic = None
@@ -425,7 +445,7 @@ def main():
     sm_mhz = clk["sm_mhz"] or float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12  # Tops/s at the sampled clock
     upd_ops = mean_dk * n_normals_update * alu_ops_per_normal / (per["update"] * 1e-3) / 1e12
-    bytes_per_step = d * (wl.n_members * 6 + 6 + 10)
+    bytes_per_step = d * ((wl.n_members // 2) * 8 + 8 + 12 if dual else wl.n_members * 6 + 6 + 10)
     value = job_throughput(world, d, args.steps, ms * 1e-3)
     e2e = job_throughput(world, d, args.e2e_steps, e2e_s)
     launches = sum(counts.values())
@@ -442,10 +462,10 @@ def main():
             ("perturb_pair" if paired else "perturb"): {
                 "ms": per["perturb"], "launches": counts["perturb"], "GB/s": achieved, "frac_hbm": achieved / hbm},
             "restore": {"ms": per["restore"], "launches": counts["restore"],
-                        "GB/s": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9,
-                        "frac_hbm": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9 / hbm},
+                        "GB/s": restore_bytes / (per["restore"] * 1e-3) / 1e9,
+                        "frac_hbm": restore_bytes / (per["restore"] * 1e-3) / 1e9 / hbm},
             "update_fused_commit": {"ms": per["update"], "launches": counts["update"],
-                                    "GB/s": 10.0 * mean_dk / (per["update"] * 1e-3) / 1e9,
+                                    "GB/s": update_bytes / (per["update"] * 1e-3) / 1e9,
                                     "bound": "alu", "achieved_Tops": upd_ops, "peak_Tops": alu_peak,
                                     "frac_alu": upd_ops / alu_peak,
                                     "ops_per_normal": alu_ops_per_normal, "normals_per_elem": n_normals_update},
@@ -453,7 +473,7 @@ def main():
             **({"perturb_partner": {"ms": per["partner"], "launches": counts["partner"],
                                     "GB/s": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9,
                                     "frac_hbm": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9 / hbm}}
-               if paired else {}),
+               if "partner" in per else {}),
         },
         "clocks": clk,
         "e2e": {"value": e2e, "unit": "params/s", "h2d_bytes_per_step": wl.K * wl.n_members * 4,
@@ -679,7 +699,7 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
     K, chunk = 4, 65536
     layout = copes.Layout(wl.numel)
     d = wl.d
-    arena = make_arena(copes, torch, wl, layout)
+    arena = make_arena(copes, torch, wl, layout, dual=args.weights == "dual")
     cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping="zscore",
                       convention=copes.COEF_PAPER, dimension_aware=True)
     total = args.warmup + args.steps
@@ -688,8 +708,12 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
     # each step's partition is built on a side stream while the previous step runs
     parts = es.ChunkPrefetcher(layout, K, lambda s: 1000 + s, chunk=chunk, tile_size=args.tile)
     # random chunks spread every subspace over the arena: one partner buffer covers it
-    partner = None if args.no_partner else es.Partner(
-        torch.empty(layout.d_pad, dtype=arena.w.dtype, device="cuda"), 0)
+    if args.weights == "dual":
+        partner = es.Partner.second_copy(arena)
+    elif args.weights == "partner":
+        partner = es.Partner(torch.empty(layout.d_pad, dtype=arena.w.dtype, device="cuda"), 0)
+    else:
+        partner = None
 
     def step(s, events=None):
         subs = parts.take(s, events=events)
@@ -730,7 +754,7 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
     # the update's roofline is the slower of its ALU and HBM bounds
     t_alu = 28.0 * P * mean_dk / (alu_peak * 1e12)
     t_hbm = 10.0 * mean_dk / (hbm * 1e9)
-    paired = "partner" in per
+    paired = args.weights != "single"
     perturb_gbs = (8.0 if paired else 6.0) * mean_dk / (per["perturb"] * 1e-3) / 1e9
     value = job_throughput(world, d, args.steps, ms * 1e-3)
     out = {
@@ -741,7 +765,8 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
                                "(65,536) resampled per step, N=32 antithetic (N_k=8), dimension-aware sigma_k, "
                                "joint z-score, coefficient alpha/N_k",
                    "params": d, "K": K, "N": wl.n_members, "chunk": chunk, "sigma": wl.sigma, "alpha": wl.alpha,
-                   "tile": args.tile, "l2": "inputs larger than L2, no flush"},
+                   "tile": args.tile, "working_weights": WEIGHTS_MODES[args.weights],
+                   "l2": "inputs larger than L2, no flush"},
         "roofline": {"bound": "hbm", "kernel": "perturb_pair" if paired else "perturb", "achieved": perturb_gbs,
                      "peak": hbm, "unit": "GB/s", "frac": perturb_gbs / hbm, "traffic": None,
                      "peak_source": "measured"},
@@ -752,7 +777,8 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
             ("perturb_pair" if paired else "perturb"): {"ms": per["perturb"], "launches": counts["perturb"],
                                                         "GB/s": perturb_gbs, "frac_hbm": perturb_gbs / hbm},
             **({"perturb_partner": {"ms": per["partner"], "launches": counts["partner"],
-                                    "GB/s": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9}} if paired else {}),
+                                    "GB/s": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9}}
+               if "partner" in per else {}),
             "restore": {"ms": per["restore"], "launches": counts["restore"],
                         "GB/s": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9},
             "update_fused_commit": {"ms": per["update"], "launches": counts["update"], "Tops": upd_tops,

@@ -75,12 +75,19 @@ enum {
 
 /* ------------------------------------------------------------------------- data types */
 
-/* The flat parameter arena. */
+/* The flat parameter arena.
+ * w2 (optional, NULL for none) is a second working-weight buffer of the same dtype and
+ * size, for evaluating the two members of an antithetic pair on two copies of the model:
+ * copes_perturb_pair with partner = w2, partner_base = 0, partner_len = n_alloc writes
+ * member 2j's weights to w and member 2j+1's to w2 in one pass.  Restore, commit, the
+ * fused update's commit and init then write the context to w2 as well as w, so outside
+ * the live subspace both buffers always hold the context.  Perturbs write w only. */
 typedef struct {
   void *w;          /* device: working weights, n_alloc elements of dtype              */
   float *master;    /* device: fp32 master theta, n_alloc elements                     */
   uint64_t n_alloc; /* elements in each buffer; every subspace index must be < n_alloc */
   int dtype;        /* COPES_BF16 or COPES_FP32 (the dtype of w)                       */
+  void *w2;         /* device, optional: second working buffer (16-byte aligned), or NULL */
 } copes_params;
 
 /* A subspace S (Eq. 7 / Eq. 8: the support of P_k).

@@ -42,7 +42,7 @@ class CopesError(RuntimeError):
 
 class Params(ctypes.Structure):
     _fields_ = [("w", ctypes.c_void_p), ("master", ctypes.c_void_p), ("n_alloc", ctypes.c_uint64),
-                ("dtype", ctypes.c_int)]
+                ("dtype", ctypes.c_int), ("w2", ctypes.c_void_p)]
 
 
 class Subspace(ctypes.Structure):
@@ -204,14 +204,22 @@ class Layout:
 
 # ----------------------------------------------------------------------------- arena
 class Arena:
-    """The flat parameter arena: working weights w (bf16 or fp32) and the fp32 master."""
+    """The flat parameter arena: working weights w (bf16 or fp32) and the fp32 master, and
+    optionally a second working buffer w2 (copes_params.w2) that restore, commit and init
+    keep equal to w outside the live member's perturbation.  `live` is the working buffer
+    that holds the member being evaluated (w, or w2 for a pair's second member when w2
+    serves as the partner buffer)."""
 
-    def __init__(self, w: torch.Tensor, master: torch.Tensor):
+    def __init__(self, w: torch.Tensor, master: torch.Tensor, w2: Optional[torch.Tensor] = None):
         assert w.is_cuda and master.is_cuda and w.is_contiguous() and master.is_contiguous()
         assert master.dtype == torch.float32 and w.numel() == master.numel()
-        self.w, self.master = w, master
+        if w2 is not None:
+            assert w2.is_cuda and w2.is_contiguous() and w2.dtype == w.dtype and w2.numel() == w.numel()
+        self.w, self.master, self.w2 = w, master, w2
+        self.live = w
         dt = {torch.bfloat16: BF16, torch.float32: FP32}[w.dtype]
-        self.params = Params(w.data_ptr(), master.data_ptr(), w.numel(), dt)
+        self.params = Params(w.data_ptr(), master.data_ptr(), w.numel(), dt,
+                             None if w2 is None else w2.data_ptr())
 
     @classmethod
     def empty(cls, n: int, dtype=torch.bfloat16, device="cuda"):

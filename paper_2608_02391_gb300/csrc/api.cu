@@ -46,6 +46,9 @@ int check_params(const copes_params *p, const char *who) {
                 p->dtype);
   if (!aligned(p->w, 16) || !aligned(p->master, 16))
     return fail(COPES_ERR_ALIGNMENT, "%s: w and master must be 16-byte aligned", who);
+  if (p->w2 && !aligned(p->w2, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: w2 must be 16-byte aligned", who);
+  if (p->w2 && (p->w2 == p->w || p->w2 == (void *)p->master))
+    return fail(COPES_ERR_INVALID_ARG, "%s: w2 must be a buffer of its own", who);
   if (p->n_alloc == 0) return fail(COPES_ERR_SIZE, "%s: n_alloc is 0", who);
   return COPES_OK;
 }
@@ -138,6 +141,7 @@ int launch_status(cudaError_t e, const char *who) {
 ElemArgs elem_args(const copes_params *p, const copes_subspace *S) {
   ElemArgs a{};
   a.w = p->w;
+  a.w2 = p->w2;
   a.master = p->master;
   a.n_alloc = p->n_alloc;
   if (S->kind == COPES_SUBSPACE_TILES) {
@@ -707,6 +711,7 @@ int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
   UpdateArgs a{};
   if ((rc = fill_update_members(a, n_members, noise_id, sign, fitness, n_noise, seeds, coef, who))) return rc;
   a.w = p->w;
+  a.w2 = p->w2;
   a.master = p->master;
   a.n_alloc = p->n_alloc;
   if (S->kind == COPES_SUBSPACE_TILES) {

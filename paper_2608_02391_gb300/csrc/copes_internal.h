@@ -93,6 +93,7 @@ struct ScaledCoeffs {
 
 struct ElemArgs {
   void *w;
+  void *w2;  // second working buffer (copes_params.w2) or NULL: restore / commit / init write both
   float *master;
   uint64_t n_alloc;
   const uint64_t *tiles;
@@ -127,6 +128,7 @@ enum ElemOp {
 
 struct UpdateArgs {
   void *w;
+  void *w2;  // second working buffer or NULL: the fused commit writes both
   float *master;
   uint64_t n_alloc;
   const uint64_t *tiles;

@@ -31,6 +31,11 @@ __device__ __forceinline__ float index_noise(uint64_t g, uint32_t tag, uint32_t 
 template <int OP>
 constexpr uint32_t op_tag() { return OP == kOpInit ? COPES_TAG_INIT : COPES_TAG_NOISE; }
 
+// Ops whose values are the context (restore / commit, init) go to the second working
+// buffer too; perturbations go to w only.
+template <int OP>
+constexpr bool writes_context() { return OP == kOpRestore || OP == kOpInit; }
+
 // perturb: v = theta + a eps;  init: v = b + a eps;  restore: v = theta;  perturb pair:
 // v = theta + a eps and the partner's vp = theta - a eps.  (q_lo, q_hi) is the group's
 // Philox counter g4 >> 2.  Coefficients scaled by -a are the exact negatives of those
@@ -91,6 +96,7 @@ __device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b,
       }
       if (OP == kOpInit) st_stream_f4(mt + o, make_float4(v[0], v[1], v[2], v[3]));
       WStore<WT>::full(a.w, b + o, v);
+      if (writes_context<OP>() && a.w2) WStore<WT>::full(a.w2, b + o, v);
       if (OP == kOpPerturbPair) WStore<WT>::full(a.partner, b + o - a.partner_base, vp);
     }
   }
@@ -131,6 +137,7 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
       if (full[i]) {
         if (OP == kOpInit) st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
         WStore<WT>::full(a.w, g4, v);
+        if (writes_context<OP>() && a.w2) WStore<WT>::full(a.w2, g4, v);
         if (OP == kOpPerturbPair) WStore<WT>::full(a.partner, g4 - a.partner_base, vp);
       } else {
 #pragma unroll
@@ -139,6 +146,7 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
           if (g >= b && g < e) {
             if (OP == kOpInit) master[g] = v[k];
             WStore<WT>::one(a.w, g, v[k]);
+            if (writes_context<OP>() && a.w2) WStore<WT>::one(a.w2, g, v[k]);
             if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, g - a.partner_base, vp[k]);
           }
         }
@@ -294,6 +302,7 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
           else master[g[u]] = v;
         }
         WStore<WT>::one(a.w, (uint64_t)g[u], v);
+        if (writes_context<OP>() && a.w2) WStore<WT>::one(a.w2, (uint64_t)g[u], v);
         if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, (uint64_t)g[u] - a.partner_base, vp);
       }
     }
@@ -393,7 +402,10 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
         float v[4] = {__fmaf_rn(a.coef, acc[i][0], t.x), __fmaf_rn(a.coef, acc[i][1], t.y),
                       __fmaf_rn(a.coef, acc[i][2], t.z), __fmaf_rn(a.coef, acc[i][3], t.w)};
         st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
-        if (COMMIT) WStore<WT>::full(a.w, g4, v);
+        if (COMMIT) {
+          WStore<WT>::full(a.w, g4, v);
+          if (a.w2) WStore<WT>::full(a.w2, g4, v);
+        }
       } else {
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -401,7 +413,10 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
           if (g >= b && g < e) {
             const float v = __fmaf_rn(a.coef, acc[i][k], master[g]);
             master[g] = v;
-            if (COMMIT) WStore<WT>::one(a.w, g, v);
+            if (COMMIT) {
+              WStore<WT>::one(a.w, g, v);
+              if (a.w2) WStore<WT>::one(a.w2, g, v);
+            }
           }
         }
       }
@@ -498,7 +513,10 @@ __global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_con
         float *th = GATH ? &gath[first + p0 + kThreads * u] : &master[g[u]];
         const float v = __fmaf_rn(a.coef, acc[u], *th);
         *th = v;
-        if (COMMIT) WStore<WT>::one(a.w, (uint64_t)g[u], v);
+        if (COMMIT) {
+          WStore<WT>::one(a.w, (uint64_t)g[u], v);
+          if (a.w2) WStore<WT>::one(a.w2, (uint64_t)g[u], v);
+        }
       }
     }
   });

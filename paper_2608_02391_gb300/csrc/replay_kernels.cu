@@ -220,6 +220,7 @@ __global__ void __launch_bounds__(kThreads) replay_elem_kernel(const __grid_cons
         if (OP == kOpInit) master[g[u]] = v;
       }
       WStore<WT>::one(a.w, g[u], v);
+      if ((OP == kOpRestore || OP == kOpInit) && a.w2) WStore<WT>::one(a.w2, g[u], v);
       if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, g[u] - a.partner_base, vp);
     }
   }, [] {});
@@ -276,7 +277,10 @@ __global__ void __launch_bounds__(kThreads) replay_update_kernel(const __grid_co
       if (!ok[u]) continue;
       const float v = __fmaf_rn(a.coef, acc[u], master[g[u]]);
       master[g[u]] = v;
-      if (COMMIT) WStore<WT>::one(a.w, g[u], v);
+      if (COMMIT) {
+        WStore<WT>::one(a.w, g[u], v);
+        if (a.w2) WStore<WT>::one(a.w2, g[u], v);
+      }
     }
   }, [] {});
 }

@@ -50,9 +50,19 @@ class ESConfig:
 class Partner:
     """Buffer for the antithetic partner's weights (copes_perturb_pair): element g of the
     arena at buf[g - base], in the working dtype.  Partner.covering(arena, subs) sizes one
-    for every element of `subs`."""
+    for every element of `subs`.  in_place: the buffer is the arena's second working
+    buffer w2 (Partner.second_copy), so the partner member is evaluated there directly and
+    nothing is copied."""
     buf: torch.Tensor
     base: int
+    in_place: bool = False
+
+    @classmethod
+    def second_copy(cls, arena: copes.Arena) -> "Partner":
+        """The arena's second working buffer as the partner: member 2j is evaluated on w,
+        member 2j + 1 on w2."""
+        assert arena.w2 is not None, "the arena has no second working buffer"
+        return cls(arena.w2, 0, True)
 
     @classmethod
     def covering(cls, arena: copes.Arena, subs: Sequence[copes.SubspaceHandle]) -> "Partner":
@@ -75,22 +85,30 @@ def perturb_members(arena: copes.Arena, sub: copes.SubspaceHandle, members: Sequ
                     seeds, s_k: float, live: Callable[[int], None], partner: Optional[Partner] = None,
                     events: Optional[dict] = None) -> None:
     """Perturbs each member of `members` in order (Eq. 8) and calls live(i) while member i's
-    perturbation is in place.  With a partner buffer, a member whose successor shares its
-    noise vector with the opposite sign (an antithetic pair) is perturbed by
-    copes_perturb_pair, and the successor's weights are then copied in from the buffer:
-    one noise generation per pair, bit-identical weights."""
+    perturbation is in place (in arena.live).  With a partner buffer, a member whose
+    successor shares its noise vector with the opposite sign (an antithetic pair) is
+    perturbed by copes_perturb_pair, and the successor's weights are then copied in from
+    the buffer, or, for an in-place partner (the arena's w2), evaluated there: one noise
+    generation per pair, bit-identical weights."""
     staged = None  # the member whose weights the partner buffer holds
     for pos, i in enumerate(members):
         nxt = members[pos + 1] if pos + 1 < len(members) else None
         seed, ss = int(seeds[nid[i]]), float(sign[i]) * s_k
-        if staged == i:
+        where = None if arena is None else arena.w
+        if staged == i and partner.in_place:
+            where = partner.buf
+        elif staged == i:
             _timed(events, "partner", lambda: copes.perturb_partner(arena, sub, partner.buf, partner.base))
         elif partner is not None and nxt is not None and nid[nxt] == nid[i] and sign[nxt] == -sign[i]:
             _timed(events, "perturb", lambda: copes.perturb_pair(arena, sub, seed, ss, partner.buf, partner.base))
             staged = nxt
         else:
             _timed(events, "perturb", lambda: copes.perturb(arena, sub, seed, ss))
+        if arena is not None:
+            arena.live = where
         live(i)
+    if arena is not None:
+        arena.live = arena.w
 
 
 def sigma_k(cfg: ESConfig, d: int, d_k: int) -> float:

@@ -271,3 +271,15 @@ def test_partner_buffer_arguments_are_rejected_before_any_launch(lib):
     assert partner(ctypes.byref(p), ctypes.byref(bad), fake, 0, 1000, None) == copes.ERR_INVALID_ARG
     q = copes.Params(fake, fake + 4, 1000, copes.BF16)  # misaligned master
     assert partner(ctypes.byref(q), ctypes.byref(s), fake, 0, 1000, None) == copes.ERR_ALIGNMENT
+
+
+def test_second_working_buffer_is_validated(lib):
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    s = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
+    p = copes.Params(fake, fake + 64, 100, copes.BF16, fake + 8)  # misaligned w2
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_ALIGNMENT
+    p = copes.Params(fake, fake + 64, 100, copes.BF16, fake)  # w2 aliases w
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
+    p = copes.Params(fake, fake + 64, 100, copes.BF16, fake + 64)  # w2 aliases master
+    assert lib.copes_context_commit(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG

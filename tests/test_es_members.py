@@ -54,3 +54,18 @@ def test_a_slice_that_splits_a_pair(calls):
     live = run(calls, es.member_slice(1, 3, 8), nid, sign, es.Partner(None, 0))
     assert live == [3, 4, 5]
     assert calls == [("perturb", 101, -0.5), ("pair", 102, 0.5, 0), ("partner", 0)]
+
+
+def test_in_place_partner_evaluates_the_second_member_on_w2(calls):
+    """With the arena's second working buffer as the partner, member 2j + 1 is evaluated on
+    w2: no copy, and arena.live points at the buffer that holds the live member."""
+    from types import SimpleNamespace
+    arena = SimpleNamespace(w="w", w2="w2", live="w")
+    nid, sign, P = copes.member_table(6, copes.ANTITHETIC)
+    seeds = np.arange(100, 103, dtype=np.uint64)
+    seen = []
+    es.perturb_members(arena, None, range(6), nid, sign, seeds, 0.5, lambda i: seen.append((i, arena.live)),
+                       es.Partner("w2", 0, True))
+    assert seen == [(0, "w"), (1, "w2"), (2, "w"), (3, "w2"), (4, "w"), (5, "w2")]
+    assert calls == [("pair", 100, 0.5, 0), ("pair", 101, 0.5, 0), ("pair", 102, 0.5, 0)]
+    assert arena.live == "w"

@@ -197,3 +197,77 @@ def test_sync_step_with_partner_buffer_is_bit_identical(copes):
         out.append((bits(arena.w), arena.master.cpu().numpy().view(np.uint32)))
     copes.check()
     assert np.array_equal(out[0][0], out[1][0]) and np.array_equal(out[0][1], out[1][1])
+
+
+# ---------------------------------------------------- a second working buffer (w2)
+@pytest.mark.parametrize("kind", ["tiles:1000", "indices", "replay"])
+def test_second_buffer_receives_the_context_only(copes, kind):
+    """With copes_params.w2 set, restore, commit, the fused update's commit and init write
+    the same values to w2 as to w (on S only); perturbs leave w2 alone."""
+    theta = theta_np()
+    w_a, w_b = canary(N_ALLOC, torch.bfloat16, 9), canary(N_ALLOC, torch.bfloat16, 10)
+    dual = copes.Arena(w_a, torch.from_numpy(theta.copy()).cuda(), w2=w_b)
+    single = copes.Arena(w_a.clone(), torch.from_numpy(theta.copy()).cuda())
+    if kind == "replay":
+        layout = copes.Layout([N_ALLOC])
+        sub = copes.hash_replay_partition(layout, 3, 11)[1]
+        inside = np.zeros(N_ALLOC, bool)
+        inside[oracle.hash_list([N_ALLOC], [0], 3, 11, 1).astype(np.int64)] = True
+    else:
+        sub = make_sub(copes, kind, RANGES, dual)
+        inside = mask_of(RANGES)
+    b0 = bits(w_b).copy()
+    copes.perturb(dual, sub, 5, 1e-3)
+    copes.perturb(single, sub, 5, 1e-3)
+    assert np.array_equal(bits(dual.w), bits(single.w)) and np.array_equal(bits(w_b), b0)
+    copes.restore(dual, sub)
+    copes.restore(single, sub)
+    got_w, got_w2 = bits(dual.w), bits(w_b)
+    assert np.array_equal(got_w, bits(single.w))
+    assert np.array_equal(got_w2[inside], got_w[inside]) and np.array_equal(got_w2[~inside], b0[~inside])
+    nid, sign, P = copes.member_table(4, copes.ANTITHETIC)
+    f = torch.tensor([1.0, -0.5, 0.25, 2.0], device="cuda")
+    for a in (dual, single):
+        copes.update(a, sub, nid, sign, f, copes.member_seeds(33, 0, 0, P), 0.1, fuse_commit=True)
+    assert np.array_equal(dual.master.cpu().numpy().view(np.uint32), single.master.cpu().numpy().view(np.uint32))
+    got_w, got_w2 = bits(dual.w), bits(w_b)
+    assert np.array_equal(got_w, bits(single.w))
+    assert np.array_equal(got_w2[inside], got_w[inside]) and np.array_equal(got_w2[~inside], b0[~inside])
+    copes.init_normal(dual, sub, 7, 0.0, 0.02)
+    assert np.array_equal(bits(w_b)[inside], bits(dual.w)[inside])
+    copes.check()
+
+
+def dual_trace(copes, es, mode, kind):
+    n = 1 << 18
+    theta = theta_np(n, 3)
+    w = torch.from_numpy(theta.copy()).cuda().to(torch.bfloat16)
+    arena = copes.Arena(w, torch.from_numpy(theta.copy()).cuda(), w2=w.clone() if mode == "dual" else None)
+    layout = copes.Layout([n // 2, n // 2 - 100])
+    subs = (es.build_subspaces(layout, "contiguous", 3, tile_size=4096) if kind == "tiles"
+            else copes.hash_replay_partition(layout, 3, 5))
+    partner = es.Partner.second_copy(arena) if mode == "dual" else None
+    cfg = es.ESConfig(n_members=8, sigma=1e-3, alpha=5e-4)
+    rng = np.random.default_rng(1)
+    trace = []
+    for k, sub in enumerate(subs):
+        r = torch.from_numpy(rng.standard_normal(8).astype(np.float32)).cuda()
+
+        def ev(i):  # what a rollout would see: the live buffer's bits
+            trace.append(int(arena.live.view(torch.int16).to(torch.int64).mul(i + 1).sum()))
+
+        es.round_robin_visit(arena, sub, k, 0, cfg, n, r, evaluate=ev, partner=partner)
+    copes.check()
+    return trace, arena
+
+
+@pytest.mark.parametrize("kind", ["tiles", "replay"])
+def test_visit_on_two_working_buffers_is_bit_identical(copes, kind):
+    """Members 2j on w and 2j + 1 on w2: every member sees the weights it sees with one
+    buffer, and after the visits w, w2 and the master equal the one-buffer run's."""
+    from paper_2608_02391_gb300 import es
+    t0, a0 = dual_trace(copes, es, "single", kind)
+    t1, a1 = dual_trace(copes, es, "dual", kind)
+    assert t0 == t1 and len(t0) == 24
+    assert np.array_equal(bits(a1.w), bits(a0.w)) and np.array_equal(bits(a1.w2), bits(a0.w))
+    assert np.array_equal(a1.master.cpu().numpy().view(np.uint32), a0.master.cpu().numpy().view(np.uint32))
