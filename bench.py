@@ -503,7 +503,14 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
     from paper_2608_02391_gb300 import workloads
     layout = copes.Layout(wl.numel, list(range(len(wl.tensors))))
     d = wl.d
-    arena = make_arena(copes, torch, wl, layout)
+    arena = make_arena(copes, torch, wl, layout, dual=args.weights == "dual")
+    # a hash subspace spreads over the whole arena: the partner is w2 or a full-size buffer
+    if args.weights == "dual":
+        partner = es.Partner.second_copy(arena)
+    elif args.weights == "partner":
+        partner = es.Partner(torch.empty(layout.d_pad, dtype=arena.w.dtype, device="cuda"), 0)
+    else:
+        partner = None
     mask_buf = None
     if args.hash_mode in ("replay", "replay-mask"):
         subs = copes.hash_replay_partition(layout, wl.K, wl.partition_seed)
@@ -524,7 +531,7 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
             if mask_buf is not None:
                 es._timed(events, "mask", lambda: copes.hash_replay_mask(arena, subs[k], mask_buf))
             es.round_robin_visit(arena, subs[k], k, s, cfg, d, rewards[s * wl.K + k], fitness_out=fitness,
-                                 events=events)
+                                 events=events, partner=partner)
 
     for s in range(args.warmup):
         step(s)
@@ -561,8 +568,10 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
     # replay adds the membership hash of every element (one Philox call = 80 ops per 4)
     upd_ops = 28.0 * P * mean_dk + (20.0 * d if replay else 0.0)
     upd_tops = upd_ops / (per["update"] * 1e-3) / 1e12
-    # perturb: 6 B per member (read fp32, write bf16), plus 8 B of index per member for lists
-    pb = (6.0 if replay else 14.0) * mean_dk
+    # perturb: 6 B per member (read fp32, write bf16), 8 B for a pair perturb (two bf16
+    # writes), plus 8 B of index per member for lists
+    lists = args.hash_mode in ("lists", "gathered")
+    pb = ((8.0 if partner is not None else 6.0) + (8.0 if lists else 0.0)) * mean_dk
     value = job_throughput(world, d, args.steps, ms * 1e-3)
     out = {
         "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
@@ -573,15 +582,17 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
                                + f", K=16 hash subspaces ({args.hash_mode}), N=64 antithetic, one sweep per step",
                    "params": d, "K": wl.K, "N": wl.n_members, "sigma": wl.sigma, "alpha": wl.alpha,
                    "shaping": wl.shaping, "hash_mode": args.hash_mode, "partition_seed": wl.partition_seed,
-                   "l2": "inputs larger than L2, no flush"},
+                   "working_weights": WEIGHTS_MODES[args.weights], "l2": "inputs larger than L2, no flush"},
         "roofline": {"bound": "alu", "kernel": "update", "achieved": upd_tops, "peak": alu_peak,
                      "unit": "Tops/s", "frac": upd_tops / alu_peak, "traffic": None,
                      "peak_source": "SMs x 128 lanes x sampled SM clock",
                      "algorithmic_ops_per_launch": upd_ops},
         "kernels": {
-            "perturb": {"ms": per["perturb"], "launches": counts["perturb"],
-                        "GB/s": pb / (per["perturb"] * 1e-3) / 1e9,
-                        "frac_hbm": pb / (per["perturb"] * 1e-3) / 1e9 / hbm},
+            ("perturb_pair" if partner is not None else "perturb"): {
+                "ms": per["perturb"], "launches": counts["perturb"], "GB/s": pb / (per["perturb"] * 1e-3) / 1e9,
+                "frac_hbm": pb / (per["perturb"] * 1e-3) / 1e9 / hbm},
+            **({"perturb_partner": {"ms": per["partner"], "launches": counts["partner"]}}
+               if "partner" in per else {}),
             "restore": {"ms": per["restore"], "launches": counts["restore"]},
             "update_fused_commit": {"ms": per["update"], "launches": counts["update"], "Tops": upd_tops,
                                     "frac_alu": upd_tops / alu_peak},
