@@ -645,11 +645,14 @@ def run_backup(args, wl, copes, es, torch, rank, world, local):
     total = args.warmup + args.steps
     rewards = torch.from_numpy(workloads.reward_stream(wl, total * wl.K)).cuda()
     fitness = torch.empty(wl.n_members, dtype=torch.float32, device="cuda")
+    # the backup mode keeps one working copy: antithetic pairs read the backup once into a
+    # device partner buffer as wide as the widest subspace (unless --weights single)
+    partners = [None] * wl.K if args.weights == "single" else es.Partner.per_subspace(arena, subs)
 
     def step(s, events=None):
         for k in range(wl.K):
             es.backup_visit(arena, subs[k], k, s, cfg, d, rewards[s * wl.K + k], fitness_out=fitness,
-                            events=events)
+                            events=events, partner=partners[k])
 
     for s in range(args.warmup):
         step(s)
@@ -678,10 +681,15 @@ def run_backup(args, wl, copes, es, torch, rank, world, local):
     for name, hb in host_bytes.items():
         gbs = hb * mean_dk / (per[name] * 1e-3) / 1e9
         ref = link["d2h"] if name == "save" else link["h2d"]
-        kern[name] = {"ms": per[name], "launches": counts[name], "host_link_GB/s": gbs, "frac_link": gbs / ref}
+        label = "perturb_pair" if name == "perturb" and partners[0] is not None else name
+        kern[label] = {"ms": per[name], "launches": counts[name], "host_link_GB/s": gbs, "frac_link": gbs / ref}
+    if "partner" in per:  # device to device, no host-link traffic
+        kern["perturb_partner"] = {"ms": per["partner"], "launches": counts["partner"],
+                                   "GB/s": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9}
     kern["shape"] = {"ms": per["shape"], "launches": counts["shape"]}
     value = job_throughput(world, d, args.steps, ms * 1e-3)
-    p_gbs = kern["perturb"]["host_link_GB/s"]
+    p_name = "perturb_pair" if partners[0] is not None else "perturb"
+    p_gbs = kern[p_name]["host_link_GB/s"]
     out = {
         "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
@@ -689,8 +697,10 @@ def run_backup(args, wl, copes, es, torch, rank, world, local):
         "config": {"workload": "4B decoder-shaped bf16 set, K=8 layer blocks, N=32 antithetic, CPU weight "
                                "backup mode (bf16 context in pinned host memory, no fp32 master)",
                    "params": d, "K": wl.K, "N": wl.n_members, "tile": args.tile,
+                   "working_weights": ("one bf16 copy: member 2j+1 copied in from the pair perturb's device "
+                                       "partner buffer" if partners[0] is not None else WEIGHTS_MODES["single"]),
                    "l2": "inputs larger than L2, no flush"},
-        "roofline": {"bound": "host_link", "kernel": "perturb", "achieved": p_gbs, "peak": link["h2d"],
+        "roofline": {"bound": "host_link", "kernel": p_name, "achieved": p_gbs, "peak": link["h2d"],
                      "unit": "GB/s", "frac": p_gbs / link["h2d"], "traffic": None,
                      "peak_source": "measured pinned host->device cudaMemcpyAsync of 1 GiB"},
         "host_link_measured_GB/s": link,

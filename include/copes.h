@@ -394,6 +394,21 @@ int copes_backup_save(const copes_backup_params *p, const copes_subspace *S, cud
 int copes_backup_perturb(const copes_backup_params *p, const copes_subspace *S, uint64_t seed,
                          float signed_sigma, cudaStream_t stream);
 
+/* Antithetic pair perturb from the backup: w as copes_backup_perturb(signed_sigma) and
+ * partner[g - partner_base] = round(fma(-signed_sigma, eps_seed[g], backup[g])), the
+ * partner member's weights, from one read of the backup over the host link.  The partner
+ * buffer is device memory, bf16, with the rules of copes_perturb_pair (its device range
+ * check reports bit 16 in copes_check). */
+int copes_backup_perturb_pair(const copes_backup_params *p, const copes_subspace *S, uint64_t seed,
+                              float signed_sigma, void *partner, uint64_t partner_base,
+                              uint64_t partner_len, cudaStream_t stream);
+
+/* The partner member's perturb: w[g] = partner[g - partner_base] for g in S (device to
+ * device, no host-link traffic). */
+int copes_backup_perturb_partner(const copes_backup_params *p, const copes_subspace *S,
+                                 const void *partner, uint64_t partner_base, uint64_t partner_len,
+                                 cudaStream_t stream);
+
 /* Restore (Supp. A.8): w[g] = backup[g], bit-exact. */
 int copes_backup_restore(const copes_backup_params *p, const copes_subspace *S, cudaStream_t stream);
 

@@ -104,6 +104,8 @@ SIGNATURES = {
     "copes_scatter_master": (_I32, [_VP, _VP, _VP]),
     "copes_backup_save": (_I32, [_VP, _VP, _VP]),
     "copes_backup_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
+    "copes_backup_perturb_pair": (_I32, [_VP, _VP, _U64, _F32, _VP, _U64, _U64, _VP]),
+    "copes_backup_perturb_partner": (_I32, [_VP, _VP, _VP, _U64, _U64, _VP]),
     "copes_backup_restore": (_I32, [_VP, _VP, _VP]),
     "copes_backup_update": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _F32, _VP]),
     "copes_debug_philox": (_I32, [_U64, _U64, _U64, _U32, _U32, _VP, _VP]),
@@ -395,7 +397,7 @@ def partner_buffer(arena: Arena, subs: Sequence[SubspaceHandle]) -> Tuple[torch.
     return torch.empty(max(hi - lo, 8), dtype=arena.w.dtype, device=arena.w.device), lo
 
 
-def _partner_view(arena: Arena, partner: torch.Tensor, base: int) -> torch.Tensor:
+def _partner_view(arena, partner: torch.Tensor, base: int) -> torch.Tensor:
     assert partner.is_cuda and partner.dtype == arena.w.dtype and partner.is_contiguous()
     return partner[:max(0, min(partner.numel(), arena.w.numel() - base))]
 
@@ -525,6 +527,7 @@ class BackupArena:
         assert w.is_cuda and w.dtype == torch.bfloat16 and w.is_contiguous()
         assert backup.dtype == torch.bfloat16 and not backup.is_cuda and backup.numel() == w.numel()
         self.w, self.backup = w, backup
+        self.live = w  # the working buffer holding the member being evaluated
         self.params = BackupParams(w.data_ptr(), backup.data_ptr(), w.numel())
 
     @classmethod
@@ -542,6 +545,25 @@ def backup_perturb(arena: BackupArena, sub: SubspaceHandle, seed: int, signed_si
     S = sub.struct()
     _check(load().copes_backup_perturb(ctypes.byref(arena.params), ctypes.byref(S), seed, signed_sigma,
                                        _stream(stream)))
+
+
+def backup_perturb_pair(arena: BackupArena, sub: SubspaceHandle, seed: int, signed_sigma: float,
+                        partner: torch.Tensor, base: int = 0, stream=None) -> None:
+    """copes_backup_perturb_pair: w as backup_perturb(signed_sigma), the partner member's
+    weights (-signed_sigma) into the device buffer `partner` (element g at partner[g - base])."""
+    view = _partner_view(arena, partner, base)
+    S = sub.struct()
+    _check(load().copes_backup_perturb_pair(ctypes.byref(arena.params), ctypes.byref(S), seed, signed_sigma,
+                                            _ptr(partner), base, view.numel(), _stream(stream)))
+
+
+def backup_perturb_partner(arena: BackupArena, sub: SubspaceHandle, partner: torch.Tensor, base: int = 0,
+                           stream=None) -> None:
+    """copes_backup_perturb_partner: w[g] = partner[g - base] for g in the subspace."""
+    view = _partner_view(arena, partner, base)
+    S = sub.struct()
+    _check(load().copes_backup_perturb_partner(ctypes.byref(arena.params), ctypes.byref(S), _ptr(partner), base,
+                                               view.numel(), _stream(stream)))
 
 
 def backup_restore(arena: BackupArena, sub: SubspaceHandle, stream=None) -> None:

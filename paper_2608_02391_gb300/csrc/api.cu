@@ -540,12 +540,12 @@ int copes_perturb(const copes_params *p, const copes_subspace *S, uint64_t seed,
                          "copes_perturb");
 }
 
-static int check_partner(const copes_params *p, const void *buf, uint64_t base, uint64_t len,
+static int check_partner(uint64_t n_alloc, const void *buf, uint64_t base, uint64_t len,
                          const char *who) {
   if (!buf) return fail(COPES_ERR_INVALID_ARG, "%s: the partner buffer is NULL", who);
   if (!aligned(buf, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: the partner buffer must be 16-byte aligned", who);
   if (base % 4) return fail(COPES_ERR_ALIGNMENT, "%s: partner_base must be a multiple of 4", who);
-  if (p && (base > p->n_alloc || len > p->n_alloc - base))
+  if (base > n_alloc || len > n_alloc - base)
     return fail(COPES_ERR_SIZE, "%s: [partner_base, partner_base + partner_len) exceeds the arena", who);
   return COPES_OK;
 }
@@ -557,7 +557,7 @@ int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t 
   if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "%s: sigma is not finite", who);
   int rc = check_params(p, who);
   if (rc) return rc;
-  if ((rc = check_partner(p, partner, partner_base, partner_len, who))) return rc;
+  if ((rc = check_partner(p->n_alloc, partner, partner_base, partner_len, who))) return rc;
   return run_elementwise(copes::kOpPerturbPair, p, S, seed, COPES_TAG_NOISE, signed_sigma, 0.0f, stream,
                          who, Partner{partner, partner_base, partner_len});
 }
@@ -567,7 +567,7 @@ int copes_perturb_partner(const copes_params *p, const copes_subspace *S, const 
   const char *who = "copes_perturb_partner";
   int rc = check_params(p, who);
   if (rc) return rc;
-  if ((rc = check_partner(p, partner, partner_base, partner_len, who))) return rc;
+  if ((rc = check_partner(p->n_alloc, partner, partner_base, partner_len, who))) return rc;
   return run_elementwise(copes::kOpPartner, p, S, 0, 0, 0.0f, 0.0f, stream, who,
                          Partner{partner, partner_base, partner_len});
 }
@@ -737,6 +737,51 @@ int copes_backup_perturb(const copes_backup_params *p, const copes_subspace *S, 
                          float signed_sigma, cudaStream_t stream) {
   if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "copes_backup_perturb: sigma is not finite");
   return run_backup_elementwise(copes::kBackupPerturb, p, S, seed, signed_sigma, stream, "copes_backup_perturb");
+}
+
+int copes_backup_perturb_pair(const copes_backup_params *p, const copes_subspace *S, uint64_t seed,
+                              float signed_sigma, void *partner, uint64_t partner_base,
+                              uint64_t partner_len, cudaStream_t stream) {
+  const char *who = "copes_backup_perturb_pair";
+  if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "%s: sigma is not finite", who);
+  uint16_t *dev = nullptr;
+  int rc = check_backup(p, S, who, &dev);
+  if (rc) return rc;
+  if ((rc = check_partner(p->n_alloc, partner, partner_base, partner_len, who))) return rc;
+  ElemArgs a{};
+  a.w = p->w;
+  a.n_alloc = p->n_alloc;
+  a.tiles = S->tiles;
+  a.n_tiles = S->n_tiles;
+  a.seed_lo = (uint32_t)seed;
+  a.seed_hi = (uint32_t)(seed >> 32);
+  a.a = signed_sigma;
+  scaled_coeffs(signed_sigma, a.coeffs);
+  copes::philox_round_keys(a.seed_lo, a.seed_hi, a.rk);
+  a.partner = partner;
+  a.partner_base = partner_base;
+  a.partner_len = partner_len;
+  return launch_status(copes::launch_backup_elementwise(copes::kBackupPerturbPair, a, dev, stream), who);
+}
+
+int copes_backup_perturb_partner(const copes_backup_params *p, const copes_subspace *S,
+                                 const void *partner, uint64_t partner_base, uint64_t partner_len,
+                                 cudaStream_t stream) {
+  const char *who = "copes_backup_perturb_partner";
+  uint16_t *dev = nullptr;
+  int rc = check_backup(p, S, who, &dev);
+  if (rc) return rc;
+  if ((rc = check_partner(p->n_alloc, partner, partner_base, partner_len, who))) return rc;
+  ElemArgs a{};
+  a.w = p->w;
+  a.n_alloc = p->n_alloc;
+  a.tiles = S->tiles;
+  a.n_tiles = S->n_tiles;
+  a.partner = const_cast<void *>(partner);
+  a.partner_base = partner_base;
+  a.partner_len = partner_len;
+  return launch_status(copes::launch_elementwise(copes::kOpPartner, COPES_SUBSPACE_TILES, COPES_BF16, a, stream),
+                       who);
 }
 
 int copes_backup_restore(const copes_backup_params *p, const copes_subspace *S, cudaStream_t stream) {

@@ -4,6 +4,7 @@
 // counter and one 8-byte load or store of each bf16 array.
 //  save     backup[g] = w[g]
 //  perturb  w[g] = round(fma(s sigma, eps[g], backup[g]))      (Eq. 8)
+//  pair     perturb, and partner[g - base] = round(fma(-s sigma, eps[g], backup[g]))
 //  restore  w[g] = backup[g]
 //  update   t = fma(coef, sum_j w_j eps_j[g], backup[g]);  w[g] = backup[g] = round(t)
 // The perturb and update arithmetic is that of the master path with theta = backup.
@@ -46,12 +47,20 @@ __global__ void __launch_bounds__(kThreads) backup_elem_kernel(const __grid_cons
                                                                uint16_t *backup) {
   uint64_t b, e;
   if (!backup_tile(a.tiles, blockIdx.x, a.n_alloc, b, e)) return;
+  if (OP == kBackupPerturbPair && (b < a.partner_base || e - a.partner_base > a.partner_len)) {
+    if (threadIdx.x == 0) backup_flag(kErrPartnerRange);
+    return;
+  }
+  constexpr bool kPerturb = OP == kBackupPerturb || OP == kBackupPerturbPair;
   uint16_t *w = static_cast<uint16_t *>(a.w);
+  // partner element g at pw[g - partner_base]; partner_base is a multiple of 4 and at most b,
+  // so every group of the tile starts at or after it
+  uint16_t *pw = static_cast<uint16_t *>(a.partner);
   const uint16_t *src = OP == kBackupSave ? w : backup;
   uint16_t *dst = OP == kBackupSave ? backup : w;
   for (uint64_t g4 = (b & ~3ull) + 4ull * threadIdx.x; g4 < e; g4 += 4ull * kThreads) {
     const bool full = g4 >= b && g4 + 4 <= e;
-    if (OP != kBackupPerturb) {
+    if (!kPerturb) {
       if (full) {
         *reinterpret_cast<uint2 *>(dst + g4) = *reinterpret_cast<const uint2 *>(src + g4);
       } else {
@@ -68,15 +77,22 @@ __global__ void __launch_bounds__(kThreads) backup_elem_kernel(const __grid_cons
     }
     uint32_t x[4];
     philox4x32_10_rk((uint32_t)(g4 >> 2), (uint32_t)(g4 >> 34), 0u, COPES_TAG_NOISE, a.rk, x);
-    float xn[4], r[4], v[4];
+    float xn[4], r[4], v[4], vp[4];
     normal_parts4_x2(x, a.coeffs.central2, a.coeffs.tail, xn, r);  // r = s sigma R(L)
 #pragma unroll
-    for (int k = 0; k < 4; ++k) v[k] = __fmaf_rn(r[k], xn[k], th[k]);
+    for (int k = 0; k < 4; ++k) {
+      v[k] = __fmaf_rn(r[k], xn[k], th[k]);
+      vp[k] = __fmaf_rn(-r[k], xn[k], th[k]);
+    }
     if (full) {
       *reinterpret_cast<uint2 *>(w + g4) = pack4(v);
+      if (OP == kBackupPerturbPair) *reinterpret_cast<uint2 *>(pw + (g4 - a.partner_base)) = pack4(vp);
     } else {
       for (int k = 0; k < 4; ++k)
-        if (g4 + k >= b && g4 + k < e) w[g4 + k] = to_bf16_bits(v[k]);
+        if (g4 + k >= b && g4 + k < e) {
+          w[g4 + k] = to_bf16_bits(v[k]);
+          if (OP == kBackupPerturbPair) pw[g4 + k - a.partner_base] = to_bf16_bits(vp[k]);
+        }
     }
   }
 }
@@ -149,6 +165,7 @@ cudaError_t launch_backup_elementwise(int op, const ElemArgs &a, uint16_t *backu
   switch (op) {
     case kBackupSave: backup_elem_kernel<kBackupSave><<<grid, kThreads, 0, s>>>(a, backup); break;
     case kBackupPerturb: backup_elem_kernel<kBackupPerturb><<<grid, kThreads, 0, s>>>(a, backup); break;
+    case kBackupPerturbPair: backup_elem_kernel<kBackupPerturbPair><<<grid, kThreads, 0, s>>>(a, backup); break;
     default: backup_elem_kernel<kBackupRestore><<<grid, kThreads, 0, s>>>(a, backup); break;
   }
   return cudaGetLastError();

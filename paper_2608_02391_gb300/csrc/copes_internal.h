@@ -210,7 +210,9 @@ cudaError_t launch_replay_update(int dtype, const UpdateArgs &a, const ReplayArg
 cudaError_t launch_replay_mask(const ReplayArgs &r, uint64_t n_alloc, uint32_t *mask, cudaStream_t s);
 
 // CPU weight backup mode: `backup` is the device-accessible pointer of pinned host memory.
-enum BackupOp { kBackupSave = 0, kBackupPerturb = 1, kBackupRestore = 2 };
+// kBackupPerturbPair: w = round(theta + a eps) and the antithetic partner's
+// round(theta - a eps) into ElemArgs.partner, theta = the backup, read over the link once.
+enum BackupOp { kBackupSave = 0, kBackupPerturb = 1, kBackupRestore = 2, kBackupPerturbPair = 3 };
 cudaError_t launch_backup_elementwise(int op, const ElemArgs &a, uint16_t *backup, cudaStream_t s);
 cudaError_t launch_backup_update(const UpdateArgs &a, uint16_t *backup, cudaStream_t s);
 

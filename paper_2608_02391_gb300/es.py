@@ -83,13 +83,18 @@ class Partner:
 
 def perturb_members(arena: copes.Arena, sub: copes.SubspaceHandle, members: Sequence[int], nid, sign,
                     seeds, s_k: float, live: Callable[[int], None], partner: Optional[Partner] = None,
-                    events: Optional[dict] = None) -> None:
+                    events: Optional[dict] = None, backup: bool = False) -> None:
     """Perturbs each member of `members` in order (Eq. 8) and calls live(i) while member i's
     perturbation is in place (in arena.live).  With a partner buffer, a member whose
     successor shares its noise vector with the opposite sign (an antithetic pair) is
     perturbed by copes_perturb_pair, and the successor's weights are then copied in from
     the buffer, or, for an in-place partner (the arena's w2), evaluated there: one noise
-    generation per pair, bit-identical weights."""
+    generation per pair, bit-identical weights.  backup: the CPU weight backup mode's
+    calls (arena is a copes.BackupArena)."""
+    if backup:
+        perturb, pair, copy = copes.backup_perturb, copes.backup_perturb_pair, copes.backup_perturb_partner
+    else:
+        perturb, pair, copy = copes.perturb, copes.perturb_pair, copes.perturb_partner
     staged = None  # the member whose weights the partner buffer holds
     for pos, i in enumerate(members):
         nxt = members[pos + 1] if pos + 1 < len(members) else None
@@ -98,12 +103,12 @@ def perturb_members(arena: copes.Arena, sub: copes.SubspaceHandle, members: Sequ
         if staged == i and partner.in_place:
             where = partner.buf
         elif staged == i:
-            _timed(events, "partner", lambda: copes.perturb_partner(arena, sub, partner.buf, partner.base))
+            _timed(events, "partner", lambda: copy(arena, sub, partner.buf, partner.base))
         elif partner is not None and nxt is not None and nid[nxt] == nid[i] and sign[nxt] == -sign[i]:
-            _timed(events, "perturb", lambda: copes.perturb_pair(arena, sub, seed, ss, partner.buf, partner.base))
+            _timed(events, "perturb", lambda: pair(arena, sub, seed, ss, partner.buf, partner.base))
             staged = nxt
         else:
-            _timed(events, "perturb", lambda: copes.perturb(arena, sub, seed, ss))
+            _timed(events, "perturb", lambda: perturb(arena, sub, seed, ss))
         if arena is not None:
             arena.live = where
         live(i)
@@ -142,19 +147,18 @@ def backup_visit(arena: copes.BackupArena, sub: copes.SubspaceHandle, k: int, it
                  cfg: ESConfig, d: int, rewards: torch.Tensor,
                  evaluate: Optional[Callable[[int], None]] = None,
                  fitness_out: Optional[torch.Tensor] = None,
-                 events: Optional[dict] = None) -> torch.Tensor:
+                 events: Optional[dict] = None, partner: Optional[Partner] = None) -> torch.Tensor:
     """One ES iteration on subspace k in the CPU weight backup mode: save the context of S
     to the host backup, evaluate the N members perturbed from it, restore, shape, and
-    apply the update, which writes the new context to the weights and the backup."""
+    apply the update, which writes the new context to the weights and the backup.
+    `partner` (a device buffer, not in place): antithetic pairs read the backup once."""
+    assert partner is None or not partner.in_place, "the backup mode has one working copy"
     nid, sign, P = copes.member_table(cfg.n_members, cfg.pairing)
     seeds = copes.member_seeds(cfg.base_seed, iteration, k, P)
     s_k = sigma_k(cfg, d, sub.numel)
     _timed(events, "save", lambda: copes.backup_save(arena, sub))
-    for i in range(cfg.n_members):
-        _timed(events, "perturb",
-               lambda: copes.backup_perturb(arena, sub, int(seeds[nid[i]]), float(sign[i]) * s_k))
-        if evaluate is not None:
-            evaluate(i)
+    perturb_members(arena, sub, range(cfg.n_members), nid, sign, seeds, s_k,
+                    evaluate if evaluate is not None else (lambda i: None), partner, events, backup=True)
     _timed(events, "restore", lambda: copes.backup_restore(arena, sub))
     f = fitness_out if fitness_out is not None else torch.empty_like(rewards)
     _timed(events, "shape", lambda: copes.shape_fitness(rewards, cfg.shaping, out=f))

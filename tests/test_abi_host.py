@@ -283,3 +283,15 @@ def test_second_working_buffer_is_validated(lib):
     assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
     p = copes.Params(fake, fake + 64, 100, copes.BF16, fake + 64)  # w2 aliases master
     assert lib.copes_context_commit(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
+
+
+def test_backup_partner_arguments_are_rejected_before_any_launch(lib):
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    s = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
+    p = copes.BackupParams(fake + 8, fake, 1000)  # misaligned w
+    assert lib.copes_backup_perturb_pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake, 0, 1000,
+                                         None) == copes.ERR_ALIGNMENT
+    assert lib.copes_backup_perturb_pair(ctypes.byref(p), ctypes.byref(s), 1, float("nan"), fake, 0, 1000,
+                                         None) == copes.ERR_INVALID_ARG
+    assert lib.copes_backup_perturb_partner(None, ctypes.byref(s), fake, 0, 1000, None) == copes.ERR_INVALID_ARG

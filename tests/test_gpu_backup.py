@@ -113,3 +113,62 @@ def test_pageable_backup_is_rejected(copes):
     with pytest.raises(copes.CopesError) as e:
         copes.backup_save(arena, sub)
     assert e.value.code == copes.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("tile", [4096, 999])
+def test_pair_perturb_from_the_backup(copes, tile):
+    """copes_backup_perturb_pair: w as backup_perturb(+s sigma), the device partner buffer
+    as backup_perturb(-s sigma), bit for bit; the partner copy then gives the second
+    member; the backup and everything outside S stay untouched."""
+    ref, arena = make(copes), make(copes)
+    sub = copes.tiles_from_ranges(RANGES, tile_size=tile)
+    inside = inside_mask()
+    g = np.nonzero(inside)[0]
+    for a in (ref, arena):
+        copes.backup_save(a, sub)
+    torch.cuda.synchronize()
+    b0 = bits(arena.backup).copy()
+    buf = bf16_canary(N_ALLOC, 4).cuda()
+    buf0 = bits(buf).copy()
+    copes.backup_perturb(ref, sub, 21, 2e-3)
+    plus = bits(ref.w).copy()
+    copes.backup_perturb(ref, sub, 21, -2e-3)
+    minus = bits(ref.w).copy()
+    copes.backup_perturb_pair(arena, sub, 21, 2e-3, buf, 0)
+    assert np.array_equal(bits(arena.w), plus)
+    pb = bits(buf)
+    assert np.array_equal(pb[g], minus[inside])
+    out = np.ones(buf.numel(), bool)
+    out[g] = False
+    assert np.array_equal(pb[out], buf0[out])
+    copes.backup_perturb_partner(arena, sub, buf, 0)
+    assert np.array_equal(bits(arena.w), minus)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits(arena.backup), b0)
+    copes.check()
+
+
+def test_backup_visit_with_partner_buffer_is_bit_identical(copes):
+    from paper_2608_02391_gb300 import es
+    results = []
+    for use in (False, True):
+        arena = make(copes)
+        subs = [copes.tiles_from_ranges(RANGES[:2], tile_size=4096), copes.tiles_from_ranges(RANGES[2:], tile_size=999)]
+        for sub in subs:
+            copes.backup_save(arena, sub)
+        partners = es.Partner.per_subspace(arena, subs) if use else [None, None]
+        cfg = es.ESConfig(n_members=8, sigma=1e-3, alpha=5e-4)
+        rng = np.random.default_rng(2)
+        trace = []
+        for k, sub in enumerate(subs):
+            r = torch.from_numpy(rng.standard_normal(8).astype(np.float32)).cuda()
+
+            def ev(i):
+                trace.append(int(arena.live.view(torch.int16).to(torch.int64).mul(i + 1).sum()))
+
+            es.backup_visit(arena, sub, k, 0, cfg, N_ALLOC, r, evaluate=ev, partner=partners[k])
+        torch.cuda.synchronize()
+        results.append((trace, bits(arena.w).copy(), bits(arena.backup).copy()))
+    copes.check()
+    assert results[0][0] == results[1][0] and len(results[0][0]) == 16
+    assert np.array_equal(results[0][1], results[1][1]) and np.array_equal(results[0][2], results[1][2])
