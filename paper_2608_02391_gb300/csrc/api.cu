@@ -682,11 +682,18 @@ int check_backup(const copes_backup_params *p, const copes_subspace *S, const ch
 }
 
 int run_backup_elementwise(int op, const copes_backup_params *p, const copes_subspace *S, uint64_t seed,
-                           float sigma, cudaStream_t s, const char *who) {
+                           float sigma, cudaStream_t s, const char *who,
+                           const Partner &partner = Partner{}) {
   uint16_t *dev = nullptr;
   int rc = check_backup(p, S, who, &dev);
   if (rc) return rc;
+  if (op == copes::kBackupPerturbPair &&
+      (rc = check_partner(p->n_alloc, partner.buf, partner.base, partner.len, who)))
+    return rc;
   ElemArgs a{};
+  a.partner = const_cast<void *>(partner.buf);
+  a.partner_base = partner.base;
+  a.partner_len = partner.len;
   a.w = p->w;
   a.n_alloc = p->n_alloc;
   a.tiles = S->tiles;
@@ -744,24 +751,8 @@ int copes_backup_perturb_pair(const copes_backup_params *p, const copes_subspace
                               uint64_t partner_len, cudaStream_t stream) {
   const char *who = "copes_backup_perturb_pair";
   if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "%s: sigma is not finite", who);
-  uint16_t *dev = nullptr;
-  int rc = check_backup(p, S, who, &dev);
-  if (rc) return rc;
-  if ((rc = check_partner(p->n_alloc, partner, partner_base, partner_len, who))) return rc;
-  ElemArgs a{};
-  a.w = p->w;
-  a.n_alloc = p->n_alloc;
-  a.tiles = S->tiles;
-  a.n_tiles = S->n_tiles;
-  a.seed_lo = (uint32_t)seed;
-  a.seed_hi = (uint32_t)(seed >> 32);
-  a.a = signed_sigma;
-  scaled_coeffs(signed_sigma, a.coeffs);
-  copes::philox_round_keys(a.seed_lo, a.seed_hi, a.rk);
-  a.partner = partner;
-  a.partner_base = partner_base;
-  a.partner_len = partner_len;
-  return launch_status(copes::launch_backup_elementwise(copes::kBackupPerturbPair, a, dev, stream), who);
+  return run_backup_elementwise(copes::kBackupPerturbPair, p, S, seed, signed_sigma, stream, who,
+                                Partner{partner, partner_base, partner_len});
 }
 
 int copes_backup_perturb_partner(const copes_backup_params *p, const copes_subspace *S,
