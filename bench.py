@@ -54,10 +54,10 @@ FALLBACK_HBM_GBS = 6800.0
 
 # ncu DRAM bytes per element of the dominant kernel (the pair perturb, or the plain perturb
 # under --weights single; bf16) from one capture each; a figure is dropped (traffic = null)
-# when es_kernels.cu or copes_device.cuh no longer matches the hash it was taken on.
+# when the tile kernels' sources (source_sha) no longer match the hash it was taken on.
 NCU_TRAFFIC = {
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "e307f929a5d1d206",
-                     "bytes_per_elem": 7.228, "capture": "profiles/perturb_pair_4b_slice.md"},
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "d0750e65c97b81bc",
+                     "bytes_per_elem": 7.226, "capture": "profiles/perturb_pair_4b_slice.md"},
     "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "fd276ea14451ff07",
                 "bytes_per_elem": 5.414, "capture": "profiles/perturb_4b_slice.md"},
 }
@@ -133,11 +133,12 @@ def measured_peaks():
 
 
 def source_sha():
-    with open(os.path.join(ROOT, "paper_2608_02391_gb300", "csrc", "es_kernels.cu"), "rb") as fh:
-        a = fh.read()
-    with open(os.path.join(ROOT, "paper_2608_02391_gb300", "csrc", "copes_device.cuh"), "rb") as fh:
-        b = fh.read()
-    return hashlib.sha256(a + b).hexdigest()[:16]
+    """Hash of the sources the tile kernels compile from."""
+    h = hashlib.sha256()
+    for name in ("es_kernels.cu", "copes_device.cuh", "copes_internal.h", "es_common.cuh", "normal_coeffs.h"):
+        with open(os.path.join(ROOT, "paper_2608_02391_gb300", "csrc", name), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
 
 
 class ClockSampler:

@@ -93,7 +93,6 @@ struct ScaledCoeffs {
 
 struct ElemArgs {
   void *w;
-  void *w2;  // second working buffer (copes_params.w2) or NULL: restore / commit / init write both
   float *master;
   uint64_t n_alloc;
   const uint64_t *tiles;
@@ -111,6 +110,7 @@ struct ElemArgs {
   // g at partner[g - partner_base] for partner_base <= g < partner_base + partner_len
   void *partner;
   uint64_t partner_base, partner_len;
+  void *w2;  // second working buffer (copes_params.w2) or NULL: restore / commit / init write both
 };
 
 // kOpGather / kOpScatter copy theta between master and the gathered copy (INDICES only).
@@ -128,7 +128,6 @@ enum ElemOp {
 
 struct UpdateArgs {
   void *w;
-  void *w2;  // second working buffer or NULL: the fused commit writes both
   float *master;
   uint64_t n_alloc;
   const uint64_t *tiles;
@@ -146,6 +145,7 @@ struct UpdateArgs {
   uint16_t noise_member[COPES_MAX_MEMBERS];
   int8_t sign[COPES_MAX_MEMBERS];
   float *gathered;  // INDICES: theta in list order instead of master[index[p]] (or NULL)
+  void *w2;         // second working buffer or NULL: the fused commit writes both
 };
 
 // ------------------------------------------------------------------------ launchers
