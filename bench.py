@@ -58,8 +58,8 @@ FALLBACK_HBM_GBS = 6800.0
 NCU_TRAFFIC = {
     "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "d0750e65c97b81bc",
                      "bytes_per_elem": 7.226, "capture": "profiles/perturb_pair_4b_slice.md"},
-    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "fd276ea14451ff07",
-                "bytes_per_elem": 5.414, "capture": "profiles/perturb_4b_slice.md"},
+    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "d0750e65c97b81bc",
+                "bytes_per_elem": 5.418, "capture": "profiles/perturb_4b_slice.md"},
 }
 
 
