@@ -3,14 +3,18 @@
 
 Workload: 4B-parameter decoder-shaped set (36 layers, hidden 2560, MLP 9728, vocab 151936,
 tied embeddings; 4,022,468,096 parameters), bf16 working weights + fp32 master (24 GB
-resident), K = 8 layer-block subspaces, N = 32 antithetic members, sigma = 1e-3,
-alpha = 5e-4, z-score shaping, step coefficient alpha / (N sigma).
+resident, plus an 8 GB second working copy by default), K = 8 layer-block subspaces,
+N = 32 antithetic members, sigma = 1e-3, alpha = 5e-4, z-score shaping, step coefficient
+alpha / (N sigma).
 
 One step = one cooperative-coevolution cycle: for each of the 8 subspaces, rebuild its
-tile table (the partition step), 32 perturbs (one per member; rewards are seeded
-synthetic scalars, no model is evaluated), restore, fitness shaping and the fused update
-+ context commit.  Every parameter passes through 32 perturbs, one restore and one
-update per step, so value = parameters per step x steps / time.
+tile table (the partition step), perturb the 32 members (rewards are seeded synthetic
+scalars, no model is evaluated), restore, fitness shaping and the fused update + context
+commit.  Every parameter passes through 32 member perturbations, one restore and one
+update per step, so value = parameters per step x steps / time.  `--weights` picks how
+the members are materialised: `dual` (default) writes antithetic members 2j and 2j+1 to
+two working copies in one pass; `partner` keeps one copy and copies member 2j+1 in from
+a partner buffer; `single` perturbs every member from theta.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl copes|reference]
 
