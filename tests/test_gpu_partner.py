@@ -200,12 +200,13 @@ def test_sync_step_with_partner_buffer_is_bit_identical(copes):
 
 
 # ---------------------------------------------------- a second working buffer (w2)
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("kind", ["tiles:1000", "indices", "replay"])
-def test_second_buffer_receives_the_context_only(copes, kind):
+def test_second_buffer_receives_the_context_only(copes, kind, dtype):
     """With copes_params.w2 set, restore, commit, the fused update's commit and init write
     the same values to w2 as to w (on S only); perturbs leave w2 alone."""
     theta = theta_np()
-    w_a, w_b = canary(N_ALLOC, torch.bfloat16, 9), canary(N_ALLOC, torch.bfloat16, 10)
+    w_a, w_b = canary(N_ALLOC, dtype, 9), canary(N_ALLOC, dtype, 10)
     dual = copes.Arena(w_a, torch.from_numpy(theta.copy()).cuda(), w2=w_b)
     single = copes.Arena(w_a.clone(), torch.from_numpy(theta.copy()).cuda())
     if kind == "replay":
