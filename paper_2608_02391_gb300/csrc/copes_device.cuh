@@ -166,6 +166,73 @@ __device__ __forceinline__ void normals4_x2(const uint32_t (&w)[4], float (&eps)
   for (int e = 0; e < 4; ++e) eps[e] = __fmul_rn(x[e], r[e]);
 }
 
+__device__ __forceinline__ unsigned long long add_f32x2(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ unsigned long long mul_f32x2(unsigned long long a, unsigned long long b) {
+  unsigned long long d;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ unsigned long long splat_f32x2(float c) {
+  const unsigned long long b = __float_as_uint(c);
+  return (b << 32) | b;
+}
+
+// normal_parts4_x2 with every step on packed pairs: x2[p] = (x_2p, x_2p+1) and
+// r2[p] = (r_2p, r_2p+1).  Each packed op rounds like its scalar form, and x^2 - 1 is the
+// exact negative of 1 - x^2 under round-to-nearest, so the results are those of
+// normal_parts4_x2 bit for bit, at fewer issue slots.
+template <int NC, int NT>
+__device__ __forceinline__ void normal_parts4_packed(const uint32_t (&w)[4],
+                                                     const unsigned long long (&central2)[NC],
+                                                     const float (&tail)[NT],
+                                                     unsigned long long (&x2)[2],
+                                                     unsigned long long (&r2)[2]) {
+  float L[4];
+#pragma unroll
+  for (int p = 0; p < 2; ++p) {
+    const unsigned long long F = pack_f32x2(__uint_as_float((w[2 * p] & 0x007FFFFEu) | 0x40000001u),
+                                            __uint_as_float((w[2 * p + 1] & 0x007FFFFEu) | 0x40000001u));
+    x2[p] = add_f32x2(F, splat_f32x2(-3.0f));
+    float t0, t1;  // x^2 - 1 = -(1 - x^2)
+    unpack_f32x2(fma_f32x2(x2[p], x2[p], splat_f32x2(-1.0f)), t0, t1);
+    L[2 * p] = lg2_approx(-t0);
+    L[2 * p + 1] = lg2_approx(-t1);
+    const unsigned long long Lp = pack_f32x2(L[2 * p], L[2 * p + 1]);
+    unsigned long long acc = central2[NC - 1];
+#pragma unroll
+    for (int i = NC - 2; i >= 0; --i) acc = fma_f32x2(acc, Lp, central2[i]);
+    r2[p] = acc;
+  }
+  const float L_min = fminf(fminf(L[0], L[1]), fminf(L[2], L[3]));
+  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+      float r0, r1;
+      unpack_f32x2(r2[p], r0, r1);
+      if (L[2 * p] < COPES_NORMAL_L_SPLIT) r0 = tail_ratio(tail, L[2 * p]);
+      if (L[2 * p + 1] < COPES_NORMAL_L_SPLIT) r1 = tail_ratio(tail, L[2 * p + 1]);
+      r2[p] = pack_f32x2(r0, r1);
+    }
+  }
+}
+
+// eps for the four words of one Philox block as two packed pairs, with compile-time
+// coefficients: bit-identical to normals4.
+__device__ __forceinline__ void normals4_packed(const uint32_t (&w)[4], unsigned long long (&eps2)[2]) {
+  COPES_UNIT_COEFFS;
+  unsigned long long c2[COPES_NORMAL_CENTRAL_DEGREE + 1];
+#pragma unroll
+  for (int k = 0; k <= COPES_NORMAL_CENTRAL_DEGREE; ++k) c2[k] = splat_f32x2(unit_central[k]);
+  unsigned long long x2[2], r2[2];
+  normal_parts4_packed(w, c2, unit_tail, x2, r2);
+#pragma unroll
+  for (int p = 0; p < 2; ++p) eps2[p] = mul_f32x2(x2[p], r2[p]);
+}
+
 // Two standard normals from two words (of different Philox blocks), their central
 // polynomials evaluated as one packed pair with compile-time coefficients and a single
 // warp vote for the tail: bit-identical to two normal_from_word calls.

@@ -355,7 +355,9 @@ cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, c
 // weight per noise vector; every thread then regenerates all P noise vectors for its
 // groups in registers and accumulates acc = sum_j w_j eps_j (j ascending),
 // theta = fma(coef, acc, theta).
-template <typename WT, int G, bool COMMIT, bool HI0>
+// PACK: every step of the transform and the accumulation on packed fp32 pairs (the same
+// values); measured 2.5% faster with few noise vectors (P = 4) and 1% slower at P = 16.
+template <typename WT, int G, bool COMMIT, bool HI0, bool PACK>
 __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_w,
                                             const uint32_t (*s_rk)[20], uint64_t b, uint64_t e) {
   float *__restrict__ master = a.master;
@@ -363,10 +365,13 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
   const int P = a.n_noise;
   for (uint64_t base = lo + 4ull * threadIdx.x; base < e; base += 4ull * kThreads * G) {
     float acc[G][4];
+    unsigned long long acc2[G][2];  // PACK: the accumulators as pairs (acc[i][2p], acc[i][2p+1])
 #pragma unroll
-    for (int i = 0; i < G; ++i)
+    for (int i = 0; i < G; ++i) {
+      acc2[i][0] = acc2[i][1] = 0ull;
 #pragma unroll
       for (int k = 0; k < 4; ++k) acc[i][k] = 0.0f;
+    }
     const uint32_t q_lo = (uint32_t)(base >> 2);  // counter of group 0 (HI0: the whole counter)
     for (int j = 0; j < P; ++j) {
       uint32_t rk[20];
@@ -378,7 +383,6 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
       const float wj = s_w[j];
 #pragma unroll
       for (int i = 0; i < G; ++i) {
-        float eps[4];
         uint32_t w[4];
         if (HI0) {
           philox4x32_10_rk(q_lo + kThreads * i, 0u, 0u, COPES_TAG_NOISE, rk, w);
@@ -386,10 +390,25 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
           const uint64_t q = (base >> 2) + kThreads * i;
           philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, w);
         }
-        // packed central polynomial: 5% faster than scalar Horner here
-        normals4_x2(w, eps);
+        if constexpr (PACK) {
+          unsigned long long eps2[2];
+          normals4_packed(w, eps2);
 #pragma unroll
-        for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
+          for (int p = 0; p < 2; ++p) acc2[i][p] = fma_f32x2(splat_f32x2(wj), eps2[p], acc2[i][p]);
+        } else {
+          // packed central polynomial: 5% faster than scalar Horner here
+          float eps[4];
+          normals4_x2(w, eps);
+#pragma unroll
+          for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
+        }
+      }
+    }
+    if constexpr (PACK) {
+#pragma unroll
+      for (int i = 0; i < G; ++i) {
+        unpack_f32x2(acc2[i][0], acc[i][0], acc[i][1]);
+        unpack_f32x2(acc2[i][1], acc[i][2], acc[i][3]);
       }
     }
     // theta is read only now, after the noise loop, so it occupies no registers there
@@ -446,8 +465,9 @@ __global__ void __launch_bounds__(kThreads, BLOCKS) update_tiles_kernel(const __
     if (threadIdx.x == 0) flag_error(kErrTileRange);
     return;
   }
-  if ((e >> 34) == 0) update_tile<WT, G, COMMIT, true>(a, s_w, s_rk, b, e);
-  else update_tile<WT, G, COMMIT, false>(a, s_w, s_rk, b, e);
+  constexpr bool kPack = BLOCKS == kUpdateBlocksPerSMFewNoise;  // the few-noise configuration
+  if ((e >> 34) == 0) update_tile<WT, G, COMMIT, true, kPack>(a, s_w, s_rk, b, e);
+  else update_tile<WT, G, COMMIT, false, kPack>(a, s_w, s_rk, b, e);
 }
 
 // Gather form of the update: indices staged through shared memory as in
