@@ -62,27 +62,6 @@ __device__ __forceinline__ void normal_parts(uint32_t w, const float (&central)[
   }
 }
 
-// The four words of one Philox block with a single warp vote for the tail (taken by a
-// warp with probability ~6%), so the common path carries no per-normal branch.
-template <int NC, int NT>
-__device__ __forceinline__ void normal_parts4(const uint32_t (&w)[4], const float (&central)[NC],
-                                              const float (&tail)[NT], float (&x)[4],
-                                              float (&r)[4]) {
-  float L[4];
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    x[e] = lattice_x(w[e]);
-    L[e] = lg2_approx(__fmaf_rn(-x[e], x[e], 1.0f));
-    r[e] = horner(central, L[e]);
-  }
-  const float L_min = fminf(fminf(L[0], L[1]), fminf(L[2], L[3]));
-  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
-#pragma unroll
-    for (int e = 0; e < 4; ++e)
-      if (L[e] < COPES_NORMAL_L_SPLIT) r[e] = tail_ratio(tail, L[e]);
-  }
-}
-
 // Packed fp32 pairs: one fma.rn.f32x2 performs the two lanes' fp32 fmas, each rounded
 // exactly as a scalar fma, at half the instruction count.
 __device__ __forceinline__ unsigned long long pack_f32x2(float lo, float hi) {
@@ -100,8 +79,10 @@ __device__ __forceinline__ unsigned long long fma_f32x2(unsigned long long a, un
   return d;
 }
 
-// normal_parts4 with the central polynomial evaluated on two pairs of normals; central2
-// holds each coefficient twice (c, c).  Same results as normal_parts4, bit for bit.
+// The four words of one Philox block: normal_parts for each, with the central polynomial
+// evaluated on two packed pairs (central2 holds each coefficient twice, (c, c); the same
+// results bit for bit) and a single warp vote for the tail (taken by a warp with
+// probability ~6%), so the common path carries no per-normal branch.
 template <int NC, int NT>
 __device__ __forceinline__ void normal_parts4_x2(const uint32_t (&w)[4],
                                                  const unsigned long long (&central2)[NC],
@@ -140,18 +121,9 @@ __device__ __forceinline__ float normal_from_word(uint32_t w) {
   return __fmul_rn(x, r);
 }
 
-// eps for the four words of one Philox block.
-__device__ __forceinline__ void normals4(const uint32_t (&w)[4], float (&eps)[4]) {
-  COPES_UNIT_COEFFS;
-  float x[4], r[4];
-  normal_parts4(w, unit_central, unit_tail, x, r);
-#pragma unroll
-  for (int e = 0; e < 4; ++e) eps[e] = __fmul_rn(x[e], r[e]);
-}
-
-// normals4 with the central polynomial on packed fp32 pairs, its coefficients (c, c)
-// compile-time constants: bit-identical to normals4, at fewer issue slots and without
-// coefficient registers.
+// eps for the four words of one Philox block, the central polynomial on packed fp32
+// pairs with compile-time (c, c) coefficients: bit-identical to four normal_from_word
+// calls, at fewer issue slots and without coefficient registers.
 __device__ __forceinline__ void normals4_x2(const uint32_t (&w)[4], float (&eps)[4]) {
   COPES_UNIT_COEFFS;
   unsigned long long c2[COPES_NORMAL_CENTRAL_DEGREE + 1];
@@ -221,7 +193,7 @@ __device__ __forceinline__ void normal_parts4_packed(const uint32_t (&w)[4],
 }
 
 // eps for the four words of one Philox block as two packed pairs, with compile-time
-// coefficients: bit-identical to normals4.
+// coefficients: bit-identical to normals4_x2.
 __device__ __forceinline__ void normals4_packed(const uint32_t (&w)[4], unsigned long long (&eps2)[2]) {
   COPES_UNIT_COEFFS;
   unsigned long long c2[COPES_NORMAL_CENTRAL_DEGREE + 1];
