@@ -60,10 +60,10 @@ FALLBACK_HBM_GBS = 6800.0
 # under --weights single; bf16) from one capture each; a figure is dropped (traffic = null)
 # when the tile kernels' sources (source_sha) no longer match the hash it was taken on.
 NCU_TRAFFIC = {
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "dcd266fb306fbad6",
-                     "bytes_per_elem": 7.224, "capture": "profiles/perturb_pair_4b_slice.md"},
-    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "dcd266fb306fbad6",
-                "bytes_per_elem": 5.417, "capture": "profiles/perturb_4b_slice.md"},
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "35ede1dfa8ae5289",
+                     "bytes_per_elem": 7.225, "capture": "profiles/perturb_pair_4b_slice.md"},
+    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "35ede1dfa8ae5289",
+                "bytes_per_elem": 5.413, "capture": "profiles/perturb_4b_slice.md"},
 }
 
 
