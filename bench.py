@@ -797,7 +797,7 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
                      "peak": hbm, "unit": "GB/s", "frac": perturb_gbs / hbm, "traffic": None,
                      "peak_source": "measured"},
         "kernels": {
-            "partition": {"ms": per["partition"], "launches": counts["partition"],
+            "partition": {"ms": per.get("partition"), "launches": counts.get("partition", 0),
                           "note": "side-stream window, host tile building included; overlapped with "
                                   "the previous step"},
             ("perturb_pair" if paired else "perturb"): {"ms": per["perturb"], "launches": counts["perturb"],
