@@ -91,11 +91,13 @@ def parse():
     ap.add_argument("--cpu-cores", type=int, default=0,
                     help="processes of the oracle's CPU sample (0: every core this process may use)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice", "4b-backup", "4b-sync"],
+    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice", "4b-backup",
+                                                     "4b-backup-slice", "4b-sync"],
                     help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling; "
                          "4b-hash: one sweep over the 16 hash subspaces of the 4B set (N=64); "
                          "4b-hash-slice: the same on 268M parameters, for profiling; "
                          "4b-backup: the 4B step in the CPU weight backup mode (no fp32 master); "
+                         "4b-backup-slice: the same on 268M parameters, for profiling; "
                          "4b-sync: Algorithm 1 on the 4B set (K=4 random chunks resampled each step)")
     ap.add_argument("--hash-mode", default="replay", choices=["replay", "replay-mask", "lists", "gathered"],
                     help="4b-hash: subspaces replayed from the partition seed (hashing in every kernel, "
@@ -323,7 +325,7 @@ def make_arena(copes, torch, wl, layout, dual=False):
 def main():
     args = parse()
     from paper_2608_02391_gb300 import workloads
-    wl = workloads.workload("4b" if args.case in ("4b-backup", "4b-sync") else args.case)
+    wl = workloads.workload({"4b-backup": "4b", "4b-sync": "4b", "4b-backup-slice": "4b-slice"}.get(args.case, args.case))
     if args.impl == "reference":
         return run_reference(args, wl)
 
@@ -337,7 +339,7 @@ def main():
     copes.load()
     if wl.mode == "hash":
         return run_hash(args, wl, copes, es, torch, rank, world, local)
-    if args.case == "4b-backup":
+    if args.case in ("4b-backup", "4b-backup-slice"):
         return run_backup(args, wl, copes, es, torch, rank, world, local)
     if args.case == "4b-sync":
         return run_sync(args, wl, copes, es, torch, rank, world, local)
@@ -699,8 +701,10 @@ def run_backup(args, wl, copes, es, torch, rank, world, local):
         "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": "4B decoder-shaped bf16 set, K=8 layer blocks, N=32 antithetic, CPU weight "
-                               "backup mode (bf16 context in pinned host memory, no fp32 master)",
+        "config": {"workload": ("4B decoder-shaped bf16 set, K=8 layer blocks" if wl.name == "4b" else
+                                f"{wl.name}: {d} parameters in {len(wl.tensors)} tensors (profiling case), K={wl.K}")
+                               + ", N=32 antithetic, CPU weight backup mode (bf16 context in pinned host memory, "
+                                 "no fp32 master)",
                    "params": d, "K": wl.K, "N": wl.n_members, "tile": args.tile,
                    "working_weights": ("one bf16 copy: member 2j+1 copied in from the pair perturb's device "
                                        "partner buffer" if partners[0] is not None else WEIGHTS_MODES["single"]),
