@@ -272,3 +272,16 @@ def test_visit_on_two_working_buffers_is_bit_identical(copes, kind):
     assert t0 == t1 and len(t0) == 24
     assert np.array_equal(bits(a1.w), bits(a0.w)) and np.array_equal(bits(a1.w2), bits(a0.w))
     assert np.array_equal(a1.master.cpu().numpy().view(np.uint32), a0.master.cpu().numpy().view(np.uint32))
+
+
+def test_pair_on_an_empty_subspace_is_a_no_op(copes):
+    theta = theta_np(1000)
+    w = canary(1000, torch.bfloat16, 3)
+    arena = copes.Arena(w, torch.from_numpy(theta.copy()).cuda(), w2=w.clone())
+    before, before2 = bits(arena.w).copy(), bits(arena.w2).copy()
+    empty = copes.tiles_from_ranges([], tile_size=64)
+    copes.perturb_pair(arena, empty, 1, 1e-3, arena.w2, 0)
+    copes.perturb_partner(arena, empty, arena.w2, 0)
+    copes.restore(arena, empty)
+    copes.check()
+    assert np.array_equal(bits(arena.w), before) and np.array_equal(bits(arena.w2), before2)
