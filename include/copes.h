@@ -322,8 +322,9 @@ int copes_perturb(const copes_params *p, const copes_subspace *S, uint64_t seed,
  * of the noise.  partner: caller-owned device buffer of the working dtype (2 B per element
  * for bf16, 4 B for fp32), 16-byte aligned, holding global indices
  * [partner_base, partner_base + partner_len) at offsets 0 .. partner_len - 1; partner_base
- * is a multiple of 4 and the range lies inside the arena (COPES_ERR_ALIGNMENT /
- * COPES_ERR_SIZE otherwise).  An element of S outside that range is skipped and reported
+ * is a multiple of 4, the range lies inside the arena and the buffer does not overlap w
+ * (COPES_ERR_ALIGNMENT / COPES_ERR_SIZE / COPES_ERR_INVALID_ARG otherwise).  It may be the
+ * arena's second working buffer w2.  An element of S outside that range is skipped and reported
  * by copes_check (bit 16).  Entries of the buffer outside S are untouched. */
 int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t seed,
                        float signed_sigma, void *partner, uint64_t partner_base,

@@ -540,15 +540,27 @@ int copes_perturb(const copes_params *p, const copes_subspace *S, uint64_t seed,
                          "copes_perturb");
 }
 
-static int check_partner(uint64_t n_alloc, const void *buf, uint64_t base, uint64_t len,
-                         const char *who) {
+// True when the byte ranges [a, a + na) and [b, b + nb) overlap.
+static bool overlaps(const void *a, uint64_t na, const void *b, uint64_t nb) {
+  const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+  return a && b && na && nb && x < y + nb && y < x + na;
+}
+
+// The partner buffer: non-NULL, aligned, inside the arena's index range, and disjoint from
+// the working weights w it is read into (esize: bytes per working-dtype element).
+static int check_partner(uint64_t n_alloc, const void *w, uint64_t esize, const void *buf, uint64_t base,
+                         uint64_t len, const char *who) {
   if (!buf) return fail(COPES_ERR_INVALID_ARG, "%s: the partner buffer is NULL", who);
   if (!aligned(buf, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: the partner buffer must be 16-byte aligned", who);
   if (base % 4) return fail(COPES_ERR_ALIGNMENT, "%s: partner_base must be a multiple of 4", who);
   if (base > n_alloc || len > n_alloc - base)
     return fail(COPES_ERR_SIZE, "%s: [partner_base, partner_base + partner_len) exceeds the arena", who);
+  if (overlaps(buf, len * esize, w, n_alloc * esize))
+    return fail(COPES_ERR_INVALID_ARG, "%s: the partner buffer overlaps the working weights w", who);
   return COPES_OK;
 }
+
+static uint64_t elem_size(int dtype) { return dtype == COPES_BF16 ? 2 : 4; }
 
 int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t seed,
                        float signed_sigma, void *partner, uint64_t partner_base,
@@ -557,7 +569,8 @@ int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t 
   if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "%s: sigma is not finite", who);
   int rc = check_params(p, who);
   if (rc) return rc;
-  if ((rc = check_partner(p->n_alloc, partner, partner_base, partner_len, who))) return rc;
+  if ((rc = check_partner(p->n_alloc, p->w, elem_size(p->dtype), partner, partner_base, partner_len, who)))
+    return rc;
   return run_elementwise(copes::kOpPerturbPair, p, S, seed, COPES_TAG_NOISE, signed_sigma, 0.0f, stream,
                          who, Partner{partner, partner_base, partner_len});
 }
@@ -567,7 +580,8 @@ int copes_perturb_partner(const copes_params *p, const copes_subspace *S, const 
   const char *who = "copes_perturb_partner";
   int rc = check_params(p, who);
   if (rc) return rc;
-  if ((rc = check_partner(p->n_alloc, partner, partner_base, partner_len, who))) return rc;
+  if ((rc = check_partner(p->n_alloc, p->w, elem_size(p->dtype), partner, partner_base, partner_len, who)))
+    return rc;
   return run_elementwise(copes::kOpPartner, p, S, 0, 0, 0.0f, 0.0f, stream, who,
                          Partner{partner, partner_base, partner_len});
 }
@@ -688,7 +702,7 @@ int run_backup_elementwise(int op, const copes_backup_params *p, const copes_sub
   int rc = check_backup(p, S, who, &dev);
   if (rc) return rc;
   if (op == copes::kBackupPerturbPair &&
-      (rc = check_partner(p->n_alloc, partner.buf, partner.base, partner.len, who)))
+      (rc = check_partner(p->n_alloc, p->w, 2, partner.buf, partner.base, partner.len, who)))
     return rc;
   ElemArgs a{};
   a.partner = const_cast<void *>(partner.buf);
@@ -762,7 +776,7 @@ int copes_backup_perturb_partner(const copes_backup_params *p, const copes_subsp
   uint16_t *dev = nullptr;
   int rc = check_backup(p, S, who, &dev);
   if (rc) return rc;
-  if ((rc = check_partner(p->n_alloc, partner, partner_base, partner_len, who))) return rc;
+  if ((rc = check_partner(p->n_alloc, p->w, 2, partner, partner_base, partner_len, who))) return rc;
   ElemArgs a{};
   a.w = p->w;
   a.n_alloc = p->n_alloc;

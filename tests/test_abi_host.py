@@ -271,6 +271,10 @@ def test_partner_buffer_arguments_are_rejected_before_any_launch(lib):
     assert partner(ctypes.byref(p), ctypes.byref(bad), fake, 0, 1000, None) == copes.ERR_INVALID_ARG
     q = copes.Params(fake, fake + 4, 1000, copes.BF16)  # misaligned master
     assert partner(ctypes.byref(q), ctypes.byref(s), fake, 0, 1000, None) == copes.ERR_ALIGNMENT
+    # a partner buffer inside the working weights is rejected
+    r = copes.Params(fake, fake + (1 << 20), 1000, copes.BF16)
+    assert pair(ctypes.byref(r), ctypes.byref(s), 1, 1e-3, fake + 1024, 0, 100, None) == copes.ERR_INVALID_ARG
+    assert partner(ctypes.byref(r), ctypes.byref(s), fake + 1984, 0, 8, None) == copes.ERR_INVALID_ARG
 
 
 def test_second_working_buffer_is_validated(lib):
