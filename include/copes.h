@@ -338,11 +338,13 @@ int copes_perturb_partner(const copes_params *p, const copes_subspace *S, const 
                           uint64_t partner_base, uint64_t partner_len, cudaStream_t stream);
 
 /* Restore (Sec. 3.3, Supp. A.8 "CPU Weight Backup", here an on-device fp32 master):
- *   w[g] = round(theta[g]) for g in S, bit-exact; outside S untouched. */
+ *   w[g] = round(theta[g]) for g in S, bit-exact; outside S untouched.  With p->w2 set,
+ * w2[g] gets the same value. */
 int copes_restore(const copes_params *p, const copes_subspace *S, cudaStream_t stream);
 
 /* Context commit (Sec. 3.2 shared context after Eq. 13): w[g] = round(theta[g]) for
- * g in S.  Same arithmetic as copes_restore, called after copes_update. */
+ * g in S (and w2[g] with p->w2 set).  Same arithmetic as copes_restore, called after
+ * copes_update. */
 int copes_context_commit(const copes_params *p, const copes_subspace *S, cudaStream_t stream);
 
 /* Fitness shaping (Eq. 5, Eq. 12, Sec. 4.4): f = shape(r) over n rewards (device fp32),
@@ -357,14 +359,15 @@ int copes_shape_fitness(const float *rewards, int n, const int32_t *group, int m
  * All n_noise noise vectors are regenerated in registers in one pass; nothing is
  * stored.  noise_id, sign (host, n_members) and seeds (host, n_noise) are read during
  * the call; fitness is device fp32 [n_members].  fuse_commit != 0 also writes
- * w[g] = round(theta[g]) (the context commit) in the same pass. */
+ * w[g] = round(theta[g]) (the context commit; w2[g] too with p->w2 set) in the same
+ * pass. */
 int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
                  const int32_t *noise_id, const int8_t *sign, const float *fitness,
                  int n_noise, const uint64_t *seeds, float coef, int fuse_commit,
                  cudaStream_t stream);
 
 /* Synthetic initialisation (input preparation, not part of the method): for g in S,
- *   theta[g] = mean + scale * eps_seed^(INIT)[g],  w[g] = round(theta[g]). */
+ *   theta[g] = mean + scale * eps_seed^(INIT)[g],  w[g] = round(theta[g])  (and w2[g]). */
 int copes_init_normal(const copes_params *p, const copes_subspace *S, uint64_t seed,
                       float mean, float scale, cudaStream_t stream);
 
