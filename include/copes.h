@@ -56,7 +56,7 @@ enum {
   COPES_ERR_WORKSPACE = -4,    /* caller workspace or output capacity too small */
   COPES_ERR_CUDA = -5,         /* a CUDA runtime call failed (message has the text) */
   COPES_ERR_DEVICE_CHECK = -6, /* a kernel's own range check failed (see copes_check) */
-  COPES_ERR_UNSUPPORTED = -7   /* a mode this build does not implement */
+  COPES_ERR_UNSUPPORTED = -7   /* a mode this library does not implement */
 };
 
 enum { COPES_BF16 = 0, COPES_FP32 = 1 };
@@ -65,7 +65,7 @@ enum { COPES_BF16 = 0, COPES_FP32 = 1 };
 enum { COPES_TAG_NOISE = 0, COPES_TAG_INIT = 1, COPES_TAG_PARTITION = 2, COPES_TAG_SEED = 3,
        COPES_TAG_CHUNK = 4 };
 
-/* Limits of this build. */
+/* Limits of this library version. */
 enum {
   COPES_MAX_MEMBERS = 256,    /* population N per update call */
   COPES_MAX_NOISE = 256,      /* distinct noise vectors P per update call */
@@ -158,7 +158,7 @@ enum { COPES_COEF_PAPER = 0, COPES_COEF_OPENAI = 1 };
 
 /* -------------------------------------------------------------------- host utilities */
 
-/* Version string of this build (static storage). */
+/* Version string of the library (static storage). */
 const char *copes_version(void);
 
 /* Copies the calling thread's last error message into buf (NUL-terminated, truncated to
