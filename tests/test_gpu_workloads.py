@@ -373,6 +373,15 @@ def test_counters_beyond_2_34(copes):
                                        rng.integers(lo, hi, 4000)])).astype(np.int64)
     rewards = (rng.integers(0, 17, 8) / 16).astype(np.float32)
     check_visit(copes, arena, sub, sample, w, 0, 0, rewards)
+    # the antithetic pair perturb on both counter paths equals two perturbs, bit for bit
+    buf = torch.empty(hi - lo, dtype=torch.bfloat16, device="cuda")
+    copes.perturb(arena, sub, 77, 1e-3)
+    plus = arena.w[lo:hi].view(torch.int16).clone()
+    copes.perturb(arena, sub, 77, -1e-3)
+    minus = arena.w[lo:hi].view(torch.int16).clone()
+    copes.perturb_pair(arena, sub, 77, 1e-3, buf, lo)
+    assert torch.equal(arena.w[lo:hi].view(torch.int16), plus)
+    assert torch.equal(buf.view(torch.int16), minus)
     copes.check()
 
 
