@@ -25,7 +25,7 @@ def _free_port():
         return s.getsockname()[1]
 
 
-def _setup():
+def _setup(dual=False):
     import torch
     sys.path.insert(0, ROOT)
     from paper_2608_02391_gb300 import copes, es
@@ -33,7 +33,8 @@ def _setup():
     gen = torch.Generator(device="cuda")
     gen.manual_seed(0)
     master = torch.empty(N_PARAMS, device="cuda").normal_(0.0, 0.02, generator=gen)
-    arena = copes.Arena(master.to(torch.bfloat16), master)
+    w = master.to(torch.bfloat16)
+    arena = copes.Arena(w, master, w2=w.clone() if dual else None)
     c = torch.empty(N_PARAMS, device="cuda").normal_(0.0, 1.0, generator=gen)
     layout = copes.Layout([N_PARAMS])
     subs = es.build_subspaces(layout, "contiguous", K, tile_size=4096)
@@ -47,18 +48,22 @@ def _digest(torch, arena):
                           arena.w.view(torch.int16).cpu().numpy().tobytes()).hexdigest()
 
 
-def _worker(rank, world, port, out):
+def _worker(rank, world, port, out, dual):
     import torch.distributed as dist
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     dist.init_process_group("gloo", rank=rank, world_size=world)
     try:
-        torch, copes, es, arena, c, subs, cfg = _setup()
+        torch, copes, es, arena, c, subs, cfg = _setup(dual)
+        # dual: each rank evaluates its antithetic pairs on two working copies
+        partner = es.Partner.second_copy(arena) if dual else None
 
         def evaluate(i):  # the reward of the live perturbation: a linear objective
-            return float((c * arena.w.float()).sum().item())
+            return float((c * arena.live.float()).sum().item())
 
         for k in range(K):
-            es.population_visit(arena, subs[k], k, 0, cfg, N_PARAMS, evaluate)
+            es.population_visit(arena, subs[k], k, 0, cfg, N_PARAMS, evaluate, partner=partner)
+        if dual:  # both copies hold the new context
+            assert torch.equal(arena.w.view(torch.int16), arena.w2.view(torch.int16))
         copes.check()
         digest = _digest(torch, arena)
         ref = None
@@ -77,11 +82,12 @@ def _worker(rank, world, port, out):
         dist.destroy_process_group()
 
 
-def test_two_ranks_stay_bit_identical_and_match_one_process():
+@pytest.mark.parametrize("dual", [False, True])
+def test_two_ranks_stay_bit_identical_and_match_one_process(dual):
     ctx = mp.get_context("spawn")
     out = ctx.Queue()
     port = _free_port()
-    procs = [ctx.Process(target=_worker, args=(r, 2, port, out)) for r in range(2)]
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, out, dual)) for r in range(2)]
     for p in procs:
         p.start()
     res = sorted(out.get(timeout=600) for _ in procs)
