@@ -38,6 +38,14 @@ int cuda_fail(cudaError_t e, const char *what) {
 
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
+// True when the byte ranges [a, a + na) and [b, b + nb) overlap.
+static bool overlaps(const void *a, uint64_t na, const void *b, uint64_t nb) {
+  const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
+  return a && b && na && nb && x < y + nb && y < x + na;
+}
+
+static uint64_t elem_size(int dtype) { return dtype == COPES_BF16 ? 2 : 4; }
+
 int check_params(const copes_params *p, const char *who) {
   if (!p) return fail(COPES_ERR_INVALID_ARG, "%s: params is NULL", who);
   if (!p->w || !p->master) return fail(COPES_ERR_INVALID_ARG, "%s: w or master is NULL", who);
@@ -50,6 +58,12 @@ int check_params(const copes_params *p, const char *who) {
   if (p->w2 && (p->w2 == p->w || p->w2 == (void *)p->master))
     return fail(COPES_ERR_INVALID_ARG, "%s: w2 must be a buffer of its own", who);
   if (p->n_alloc == 0) return fail(COPES_ERR_SIZE, "%s: n_alloc is 0", who);
+  // the kernels read master while they write w (and w2): the three must be disjoint
+  const uint64_t wbytes = p->n_alloc * elem_size(p->dtype), mbytes = p->n_alloc * 4;
+  if (overlaps(p->w, wbytes, p->master, mbytes))
+    return fail(COPES_ERR_INVALID_ARG, "%s: w and master overlap", who);
+  if (p->w2 && (overlaps(p->w2, wbytes, p->w, wbytes) || overlaps(p->w2, wbytes, p->master, mbytes)))
+    return fail(COPES_ERR_INVALID_ARG, "%s: w2 overlaps w or master", who);
   return COPES_OK;
 }
 
@@ -540,16 +554,11 @@ int copes_perturb(const copes_params *p, const copes_subspace *S, uint64_t seed,
                          "copes_perturb");
 }
 
-// True when the byte ranges [a, a + na) and [b, b + nb) overlap.
-static bool overlaps(const void *a, uint64_t na, const void *b, uint64_t nb) {
-  const uintptr_t x = (uintptr_t)a, y = (uintptr_t)b;
-  return a && b && na && nb && x < y + nb && y < x + na;
-}
-
 // The partner buffer: non-NULL, aligned, inside the arena's index range, and disjoint from
-// the working weights w it is read into (esize: bytes per working-dtype element).
-static int check_partner(uint64_t n_alloc, const void *w, uint64_t esize, const void *buf, uint64_t base,
-                         uint64_t len, const char *who) {
+// the working weights w it is read into and from the fp32 master the pair perturb reads
+// (esize: bytes per working-dtype element; master NULL in the backup mode).
+static int check_partner(uint64_t n_alloc, const void *w, const float *master, uint64_t esize, const void *buf,
+                         uint64_t base, uint64_t len, const char *who) {
   if (!buf) return fail(COPES_ERR_INVALID_ARG, "%s: the partner buffer is NULL", who);
   if (!aligned(buf, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: the partner buffer must be 16-byte aligned", who);
   if (base % 4) return fail(COPES_ERR_ALIGNMENT, "%s: partner_base must be a multiple of 4", who);
@@ -557,10 +566,10 @@ static int check_partner(uint64_t n_alloc, const void *w, uint64_t esize, const 
     return fail(COPES_ERR_SIZE, "%s: [partner_base, partner_base + partner_len) exceeds the arena", who);
   if (overlaps(buf, len * esize, w, n_alloc * esize))
     return fail(COPES_ERR_INVALID_ARG, "%s: the partner buffer overlaps the working weights w", who);
+  if (overlaps(buf, len * esize, master, n_alloc * 4))
+    return fail(COPES_ERR_INVALID_ARG, "%s: the partner buffer overlaps the master", who);
   return COPES_OK;
 }
-
-static uint64_t elem_size(int dtype) { return dtype == COPES_BF16 ? 2 : 4; }
 
 int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t seed,
                        float signed_sigma, void *partner, uint64_t partner_base,
@@ -569,7 +578,7 @@ int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t 
   if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "%s: sigma is not finite", who);
   int rc = check_params(p, who);
   if (rc) return rc;
-  if ((rc = check_partner(p->n_alloc, p->w, elem_size(p->dtype), partner, partner_base, partner_len, who)))
+  if ((rc = check_partner(p->n_alloc, p->w, p->master, elem_size(p->dtype), partner, partner_base, partner_len, who)))
     return rc;
   return run_elementwise(copes::kOpPerturbPair, p, S, seed, COPES_TAG_NOISE, signed_sigma, 0.0f, stream,
                          who, Partner{partner, partner_base, partner_len});
@@ -580,7 +589,7 @@ int copes_perturb_partner(const copes_params *p, const copes_subspace *S, const 
   const char *who = "copes_perturb_partner";
   int rc = check_params(p, who);
   if (rc) return rc;
-  if ((rc = check_partner(p->n_alloc, p->w, elem_size(p->dtype), partner, partner_base, partner_len, who)))
+  if ((rc = check_partner(p->n_alloc, p->w, p->master, elem_size(p->dtype), partner, partner_base, partner_len, who)))
     return rc;
   return run_elementwise(copes::kOpPartner, p, S, 0, 0, 0.0f, 0.0f, stream, who,
                          Partner{partner, partner_base, partner_len});
@@ -702,7 +711,7 @@ int run_backup_elementwise(int op, const copes_backup_params *p, const copes_sub
   int rc = check_backup(p, S, who, &dev);
   if (rc) return rc;
   if (op == copes::kBackupPerturbPair &&
-      (rc = check_partner(p->n_alloc, p->w, 2, partner.buf, partner.base, partner.len, who)))
+      (rc = check_partner(p->n_alloc, p->w, nullptr, 2, partner.buf, partner.base, partner.len, who)))
     return rc;
   ElemArgs a{};
   a.partner = const_cast<void *>(partner.buf);
@@ -776,7 +785,7 @@ int copes_backup_perturb_partner(const copes_backup_params *p, const copes_subsp
   uint16_t *dev = nullptr;
   int rc = check_backup(p, S, who, &dev);
   if (rc) return rc;
-  if ((rc = check_partner(p->n_alloc, p->w, 2, partner, partner_base, partner_len, who))) return rc;
+  if ((rc = check_partner(p->n_alloc, p->w, nullptr, 2, partner, partner_base, partner_len, who))) return rc;
   ElemArgs a{};
   a.w = p->w;
   a.n_alloc = p->n_alloc;

@@ -96,9 +96,9 @@ def test_invalid_arguments_are_rejected_before_any_launch(lib):
     p = copes.Params(fake, fake + 3, 100, copes.BF16)  # misaligned master
     s = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
     assert lib.copes_perturb(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, None) == copes.ERR_ALIGNMENT
-    p = copes.Params(fake, fake, 100, 7)
+    p = copes.Params(fake, fake + (1 << 24), 100, 7)
     assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
-    p = copes.Params(fake, fake, 100, copes.BF16)
+    p = copes.Params(fake, fake + (1 << 24), 100, copes.BF16)
     bad = copes.Subspace(9, None, 0, None, 0)
     assert lib.copes_context_commit(ctypes.byref(p), ctypes.byref(bad), None) == copes.ERR_INVALID_ARG
     idx = copes.Subspace(copes.SUBSPACE_INDICES, None, 0, fake + 8, 10)
@@ -169,7 +169,7 @@ def test_hash_replay_arguments_are_rejected_before_any_copy(lib):
                                               ctypes.byref(out)) == code, (K, k, table, nbytes)
     assert lib.copes_hash_replay_subspace(ctypes.byref(L.desc), 4, 7, 1, fake, 80, None, None) == \
         copes.ERR_INVALID_ARG
-    p = copes.Params(fake, fake, 3072, copes.BF16)
+    p = copes.Params(fake, fake + (1 << 24), 3072, copes.BF16)
     def replay(**kw):
         f = dict(kind=copes.SUBSPACE_HASH_REPLAY, replay=fake, n_replay_tiles=2, n_replay_tensors=2, K=4,
                  k=1, seed=7)
@@ -223,7 +223,7 @@ def test_backup_mode_arguments_are_rejected_before_any_launch(lib):
 def test_gathered_master_arguments_are_rejected_before_any_launch(lib):
     from paper_2608_02391_gb300 import copes
     fake = 0x10000  # never dereferenced: every case below fails validation first
-    p = copes.Params(fake, fake, 100, copes.BF16)
+    p = copes.Params(fake, fake + (1 << 24), 100, copes.BF16)
     tiles = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
     tiles.gathered = fake
     assert lib.copes_perturb(ctypes.byref(p), ctypes.byref(tiles), 1, 1e-3, None) == copes.ERR_INVALID_ARG
@@ -238,7 +238,7 @@ def test_gathered_master_arguments_are_rejected_before_any_launch(lib):
 def test_replay_mask_arguments_are_rejected_before_any_launch(lib):
     from paper_2608_02391_gb300 import copes
     fake = 0x10000  # never dereferenced: every case below fails validation first
-    p = copes.Params(fake, fake, 100, copes.BF16)
+    p = copes.Params(fake, fake + (1 << 24), 100, copes.BF16)
     tiles = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
     tiles.replay_mask = fake
     assert lib.copes_perturb(ctypes.byref(p), ctypes.byref(tiles), 1, 1e-3, None) == copes.ERR_INVALID_ARG
@@ -251,30 +251,35 @@ def test_replay_mask_arguments_are_rejected_before_any_launch(lib):
 
 def test_partner_buffer_arguments_are_rejected_before_any_launch(lib):
     """copes_perturb_pair / copes_perturb_partner: the partner buffer must be non-NULL,
-    16-byte aligned, start at a multiple of 4 and lie inside the arena."""
+    16-byte aligned, start at a multiple of 4, lie inside the arena and overlap neither the
+    working weights nor the master."""
     from paper_2608_02391_gb300 import copes
     fake = 0x10000  # never dereferenced: every case below fails validation first
-    p = copes.Params(fake, fake, 1000, copes.BF16)
+    mst, buf = fake + (1 << 24), fake + (1 << 26)  # the master and a partner buffer, apart from w
+    p = copes.Params(fake, mst, 1000, copes.BF16)
     s = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
     pair, partner = lib.copes_perturb_pair, lib.copes_perturb_partner
     assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, None, 0, 1000, None) == copes.ERR_INVALID_ARG
-    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake + 2, 0, 1000, None) == copes.ERR_ALIGNMENT
-    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake, 6, 900, None) == copes.ERR_ALIGNMENT
-    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake, 8, 993, None) == copes.ERR_SIZE
-    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake, 1004, 0, None) == copes.ERR_SIZE
-    assert pair(ctypes.byref(p), ctypes.byref(s), 1, float("inf"), fake, 0, 1000, None) == copes.ERR_INVALID_ARG
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, buf + 2, 0, 1000, None) == copes.ERR_ALIGNMENT
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, buf, 6, 900, None) == copes.ERR_ALIGNMENT
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, buf, 8, 993, None) == copes.ERR_SIZE
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, buf, 1004, 0, None) == copes.ERR_SIZE
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, float("inf"), buf, 0, 1000, None) == copes.ERR_INVALID_ARG
     assert partner(ctypes.byref(p), ctypes.byref(s), None, 0, 1000, None) == copes.ERR_INVALID_ARG
-    assert partner(ctypes.byref(p), ctypes.byref(s), fake + 8, 0, 1000, None) == copes.ERR_ALIGNMENT
-    assert partner(ctypes.byref(p), ctypes.byref(s), fake, 2, 10, None) == copes.ERR_ALIGNMENT
-    assert partner(ctypes.byref(p), ctypes.byref(s), fake, 0, 1001, None) == copes.ERR_SIZE
+    assert partner(ctypes.byref(p), ctypes.byref(s), buf + 8, 0, 1000, None) == copes.ERR_ALIGNMENT
+    assert partner(ctypes.byref(p), ctypes.byref(s), buf, 2, 10, None) == copes.ERR_ALIGNMENT
+    assert partner(ctypes.byref(p), ctypes.byref(s), buf, 0, 1001, None) == copes.ERR_SIZE
     bad = copes.Subspace(9, None, 0, None, 0)
-    assert partner(ctypes.byref(p), ctypes.byref(bad), fake, 0, 1000, None) == copes.ERR_INVALID_ARG
+    assert partner(ctypes.byref(p), ctypes.byref(bad), buf, 0, 1000, None) == copes.ERR_INVALID_ARG
     q = copes.Params(fake, fake + 4, 1000, copes.BF16)  # misaligned master
-    assert partner(ctypes.byref(q), ctypes.byref(s), fake, 0, 1000, None) == copes.ERR_ALIGNMENT
+    assert partner(ctypes.byref(q), ctypes.byref(s), buf, 0, 1000, None) == copes.ERR_ALIGNMENT
     # a partner buffer inside the working weights is rejected
-    r = copes.Params(fake, fake + (1 << 20), 1000, copes.BF16)
-    assert pair(ctypes.byref(r), ctypes.byref(s), 1, 1e-3, fake + 1024, 0, 100, None) == copes.ERR_INVALID_ARG
-    assert partner(ctypes.byref(r), ctypes.byref(s), fake + 1984, 0, 8, None) == copes.ERR_INVALID_ARG
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, fake + 1024, 0, 100, None) == copes.ERR_INVALID_ARG
+    assert partner(ctypes.byref(p), ctypes.byref(s), fake + 1984, 0, 8, None) == copes.ERR_INVALID_ARG
+    # ... and so is one that overlaps the fp32 master, whose values the pair perturb reads
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, mst + 64, 0, 100, None) == copes.ERR_INVALID_ARG
+    assert pair(ctypes.byref(p), ctypes.byref(s), 1, 1e-3, mst - 192, 0, 100, None) == copes.ERR_INVALID_ARG
+    assert partner(ctypes.byref(p), ctypes.byref(s), mst + 3984, 0, 8, None) == copes.ERR_INVALID_ARG
 
 
 def test_second_working_buffer_is_validated(lib):
@@ -287,6 +292,17 @@ def test_second_working_buffer_is_validated(lib):
     assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
     p = copes.Params(fake, fake + 64, 100, copes.BF16, fake + 64)  # w2 aliases master
     assert lib.copes_context_commit(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
+    mst = fake + (1 << 24)
+    p = copes.Params(fake, fake + 64, 100, copes.BF16)  # w (200 B) runs into master
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
+    p = copes.Params(fake, mst, 100, copes.BF16, fake + 176)  # w2 starts inside w
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
+    p = copes.Params(fake, mst, 100, copes.BF16, mst - 192)  # w2 runs into master
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
+    p = copes.Params(fake, mst, 100, copes.BF16, mst + 384)  # w2 starts inside master (400 B)
+    assert lib.copes_context_commit(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
+    p = copes.Params(fake, mst, 100, copes.FP32, fake + 384)  # fp32 w is 400 B: w2 inside it
+    assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
 
 
 def test_backup_partner_arguments_are_rejected_before_any_launch(lib):
