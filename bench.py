@@ -91,9 +91,15 @@ def parse():
     ap.add_argument("--cpu-cores", type=int, default=0,
                     help="processes of the oracle's CPU sample (0: every core this process may use)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--case", default="4b", choices=["4b", "4b-slice", "4b-hash", "4b-hash-slice", "4b-backup",
-                                                     "4b-backup-slice", "4b-sync"],
-                    help="4b: the benchmark workload; 4b-slice: a 268M-parameter case for profiling; "
+    ap.add_argument("--cpu-kernels", type=int, default=1,
+                    help="1: add the oracle's single-thread per-kernel timings (tiny workload and a "
+                         "0.5B subspace sample) to cpu_baseline; 0: skip them")
+    ap.add_argument("--case", default="4b", choices=["4b", "0.5b", "8b", "4b-slice", "4b-slice-big", "4b-hash",
+                                                     "4b-hash-slice", "4b-backup", "4b-backup-slice", "4b-sync"],
+                    help="4b: the benchmark workload; 0.5b: the 0.5B set (K=8 layer groups, N=16, centred "
+                         "rank); 8b: the 8B set (K=4 type groups, N=128, sigma 5e-4; one step = one of its "
+                         "10 CC cycles); 4b-slice: a 268M-parameter case for profiling; 4b-slice-big: two "
+                         "2^28-parameter subspaces, for DRAM-traffic captures; "
                          "4b-hash: one sweep over the 16 hash subspaces of the 4B set (N=64); "
                          "4b-hash-slice: the same on 268M parameters, for profiling; "
                          "4b-backup: the 4B step in the CPU weight backup mode (no fp32 master); "
@@ -147,20 +153,35 @@ def source_sha():
     return h.hexdigest()[:16]
 
 
+def smi_gpu_id(local: int) -> str:
+    """The nvidia-smi identifier of torch device `local`.  nvidia-smi numbers GPUs
+    physically and ignores CUDA_VISIBLE_DEVICES, so the device is named by its UUID;
+    failing that, CUDA_VISIBLE_DEVICES maps the local index to the physical one."""
+    try:
+        import torch
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+        if uuid:
+            return uuid if uuid.startswith(("GPU-", "MIG-")) else "GPU-" + uuid
+    except Exception:
+        pass
+    visible = [v.strip() for v in os.environ.get("CUDA_VISIBLE_DEVICES", "").split(",") if v.strip()]
+    return visible[local] if local < len(visible) else str(local)
+
+
 class ClockSampler:
-    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
+    """nvidia-smi clocks / throttle reasons of one GPU, sampled every 200 ms while running."""
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
          "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
          "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, gpu_index: int):
-        self.gpu = gpu_index
+    def __init__(self, local: int):
+        self.gpu = smi_gpu_id(local)
         self.proc = None
 
     def __enter__(self):
         try:
             self.proc = subprocess.Popen(
-                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                ["nvidia-smi", "-i", self.gpu, f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
                  "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
@@ -193,9 +214,9 @@ class ClockSampler:
                 if val.lower() == "active":
                     reasons.add(name)
         if not sm:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0, "gpu": self.gpu}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
-                "samples": len(sm)}
+                "samples": len(sm), "gpu": self.gpu}
 
 
 # ------------------------------------------------------------------------ CPU oracle leg
@@ -219,10 +240,72 @@ def oracle_visit_sample(wl, n_sample: int, iteration: int = 0, part: int = 0):
     for i in range(N):
         oracle.perturb(w, master, sub, int(seeds[nid[i]]), float(sign[i]) * wl.sigma)
     oracle.restore(w, master, sub)
-    f = oracle.shape_fitness(rewards, oracle.SHAPE_ZSCORE)
+    f = oracle.shape_fitness(rewards, oracle_shaping(wl))
     coef = np.float32(oracle.step_coef(wl.alpha, N, wl.sigma, oracle.COEF_OPENAI))
     oracle.update(master, sub, nid, sign, f, seeds, coef, w=w)
     return time.perf_counter() - t0, n_sample
+
+
+def oracle_shaping(wl):
+    import oracle
+    return {"zscore": oracle.SHAPE_ZSCORE, "zscore_grouped": oracle.SHAPE_ZSCORE_GROUPED,
+            "centered_rank": oracle.SHAPE_CENTERED_RANK, "none": oracle.SHAPE_NONE}[wl.shaping]
+
+
+def oracle_kernel_timings(wl, n_sample: int) -> dict:
+    """The oracle's kernels one at a time on one host thread, over n_sample parameters
+    of a subspace of workload wl (bf16 working weights, its N, sigma and shaping): mean
+    time per call of perturb (two members), restore, shaping and the update with its
+    fused commit, as parameters/s and algorithmic GB/s (the GPU kernels' units)."""
+    import oracle
+    from paper_2608_02391_gb300 import workloads
+    N = wl.n_members
+    rng = np.random.default_rng(1)
+    master = (rng.standard_normal(n_sample) * 0.02).astype(np.float32)
+    w = np.zeros(n_sample, np.uint16)
+    sub = oracle.make_subspace(ranges=[(0, n_sample)])
+    nid, sign, P = oracle.member_table(N, oracle.ANTITHETIC)
+    seeds = np.array([oracle.member_seed(wl.base_seed, 0, 1, j) for j in range(P)], np.uint64)
+    rewards = workloads.reward_stream(wl, 1)[0]
+
+    def timed(fn, reps=1):
+        t0 = time.perf_counter()
+        for r in range(reps):
+            fn(r)
+        return (time.perf_counter() - t0) / reps
+
+    t_perturb = timed(lambda r: oracle.perturb(w, master, sub, int(seeds[nid[r]]), float(sign[r]) * wl.sigma), 2)
+    t_restore = timed(lambda r: oracle.restore(w, master, sub))
+    f = oracle.shape_fitness(rewards, oracle_shaping(wl))
+    t_shape = timed(lambda r: oracle.shape_fitness(rewards, oracle_shaping(wl)), 100)
+    coef = np.float32(oracle.step_coef(wl.alpha, N, wl.sigma, oracle.COEF_OPENAI))
+    t_update = timed(lambda r: oracle.update(master, sub, nid, sign, f, seeds, coef, w=w))
+    per = lambda t, b: {"ms": 1e3 * t, "params/s": n_sample / t, "GB/s": b * n_sample / t / 1e9}
+    return {"perturb": per(t_perturb, 6.0), "restore": per(t_restore, 6.0),
+            "shape": {"ms": 1e3 * t_shape, "members": N},
+            "update_fused_commit": {**per(t_update, 10.0), "normals_per_elem": P}}
+
+
+def host_cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the machine type)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() in ("Model name", "Model"):
+                name = line.split(":", 1)[1].strip()
+                if name and not name.isdigit():
+                    return name
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as fh:
+            for line in fh:
+                if line.lower().startswith(("model name", "hardware")):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.machine()
 
 
 def _oracle_part(args):
@@ -280,7 +363,7 @@ def run_reference(args, wl):
     finally:
         pool.close()
     value = tot_n / tot_t
-    sample = (f"each step: one subspace visit (N={wl.n_members} perturbs, restore, z-score shaping, "
+    sample = (f"each step: one subspace visit (N={wl.n_members} perturbs, restore, {wl.shaping} shaping, "
               f"fused update + commit) over {n} parameters per core, {pool.cores} processes on "
               f"disjoint ranges of subspace 0")
     print(json.dumps({
@@ -294,16 +377,30 @@ def run_reference(args, wl):
     }), flush=True)
 
 
+DECODER_SETS = {
+    "4b": ("4B decoder-shaped bf16 set, fp32 master, K=8 layer blocks, N=32 antithetic",
+           {"layers": 36, "hidden": 2560, "mlp": 9728, "vocab": 151936, "tied": True},
+           "24 GB or more resident per step"),
+    "0.5b": ("0.5B decoder-shaped bf16 set, fp32 master, K=8 layer groups (embeddings alone), N=16 antithetic",
+             {"layers": 24, "hidden": 896, "mlp": 4864, "vocab": 151936, "tied": True},
+             "3 GB or more resident per step"),
+    "8b": ("8B decoder-shaped bf16 set, fp32 master, K=4 subspaces by parameter type, N=128 antithetic; "
+           "one step = one cycle of the 10-cycle CC loop",
+           {"layers": 36, "hidden": 4096, "mlp": 12288, "vocab": 151936, "tied": False},
+           "49 GB or more resident per step"),
+}
+
+
 def workload_config(wl, args):
-    if wl.name != "4b":
+    if wl.name not in DECODER_SETS:
         return {"workload": f"{wl.name}: {wl.d} parameters in {len(wl.tensors)} tensors, K={wl.K}, "
                             f"N={wl.n_members} antithetic (profiling case)", "params": wl.d, "K": wl.K,
                 "N": wl.n_members, "tile": args.tile}
-    return {"workload": "4B decoder-shaped bf16 set, fp32 master, K=8 layer blocks, N=32 antithetic",
-            "params": wl.d, "layers": 36, "hidden": 2560, "mlp": 9728, "vocab": 151936, "tied": True,
+    desc, shape, resident = DECODER_SETS[wl.name]
+    return {"workload": desc, "params": wl.d, **shape,
             "K": wl.K, "N": wl.n_members, "sigma": wl.sigma, "alpha": wl.alpha, "shaping": wl.shaping,
             "tile": args.tile, "working_weights": WEIGHTS_MODES[args.weights],
-            "l2": "inputs larger than L2 (24 GB or more resident per step), no flush"}
+            "l2": f"inputs larger than L2 ({resident}), no flush"}
 
 
 # -------------------------------------------------------------------------- GPU leg
@@ -496,9 +593,18 @@ def main():
             pool.close()
         out["cpu_baseline"] = {
             "value": m / t, "unit": "params/s", "cores": pool.cores, "kind": "oracle",
+            "cpu_model": host_cpu_model(),
             "sample": f"one subspace visit (N={wl.n_members} perturbs, restore, shaping, fused update + "
                       f"commit) over {args.cpu_sample} parameters per core, {pool.cores} processes on "
                       f"disjoint ranges of subspace 0 ({m} parameters), {t:.1f} s"}
+        if args.cpu_kernels:
+            from paper_2608_02391_gb300 import workloads
+            n_k = 1 << 20
+            out["cpu_baseline"]["single_thread_kernels"] = {
+                "tiny": {"sample": f"{n_k} parameters, the tiny workload's N=8 and z-score, bf16 working "
+                                   "weights", **oracle_kernel_timings(workloads.workload("tiny"), n_k)},
+                "0.5b": {"sample": f"{n_k} parameters of a 0.5B subspace, N=16, centred rank, bf16 working "
+                                   "weights", **oracle_kernel_timings(workloads.workload("0.5b"), n_k)}}
     print(json.dumps(out), flush=True)
     if world > 1:
         dist.destroy_process_group()

@@ -193,6 +193,13 @@ def workload(name: str) -> Workload:
         ts = [Tensor(f"block{i}", 1 << 26, "attn", i) for i in range(4)]
         return Workload("4b-slice", ts, K=4, mode="groups", n_members=32, sigma=1e-3, alpha=5e-4,
                         shaping="zscore", group_of=[0, 1, 2, 3], data_seed=35)
+    if name == "4b-slice-big":
+        # traffic-capture case: two subspaces of 2^28 parameters (4 GB resident with two
+        # working copies), large enough that a kernel's unflushed L2 write-back at its end
+        # is a small fraction of its DRAM bytes
+        ts = [Tensor(f"block{i}", 1 << 28, "attn", i) for i in range(2)]
+        return Workload("4b-slice-big", ts, K=2, mode="groups", n_members=32, sigma=1e-3, alpha=5e-4,
+                        shaping="zscore", group_of=[0, 1], data_seed=35)
     if name == "4b-hash-slice":
         # profiling case of the hash workload: the same K = 16 hash partition and N = 64 on
         # 4 tensors of 2^26 parameters (1.6 GB resident)

@@ -69,3 +69,19 @@ def test_reference_arm_prints_only_on_rank_0():
     line = json.loads(res.stdout.strip().splitlines()[-1])
     assert line["impl"] == "reference" and line["unit"] == "params/s" and line["value"] > 0
     assert line["cpu_baseline"]["kind"] == "oracle" and line["e2e"]["h2d_bytes_per_step"] == 0
+
+
+def test_clock_sampler_names_the_physical_gpu(monkeypatch):
+    """nvidia-smi ignores CUDA_VISIBLE_DEVICES: without a CUDA device to give its UUID,
+    the local index is mapped through the visible-device list."""
+    sys.path.insert(0, ROOT)
+    import bench
+    import torch
+    if torch.cuda.is_available():
+        uuid = bench.smi_gpu_id(0)
+        assert uuid.startswith(("GPU-", "MIG-"))
+        return
+    monkeypatch.setenv("CUDA_VISIBLE_DEVICES", "5,GPU-1234")
+    assert bench.smi_gpu_id(0) == "5" and bench.smi_gpu_id(1) == "GPU-1234"
+    monkeypatch.setenv("CUDA_VISIBLE_DEVICES", "")
+    assert bench.smi_gpu_id(3) == "3"
