@@ -205,6 +205,85 @@ __device__ __forceinline__ void normals4_packed(const uint32_t (&w)[4], unsigned
   for (int p = 0; p < 2; ++p) eps2[p] = mul_f32x2(x2[p], r2[p]);
 }
 
+// The normals of G Philox blocks with a single warp vote for the tail: every block's central
+// polynomial on packed pairs with compile-time coefficients, then, only when some lane of
+// the warp holds a word in the tail, the tail polynomial for those words.  Each result is
+// the same function of its word as in normals4_x2, so the outputs equal G calls of it bit
+// for bit, with one vote instead of G.  eps = x * r.
+template <int G>
+__device__ __forceinline__ void normal_parts_groups_x2(const uint32_t (&w)[G][4], float (&x)[G][4],
+                                                       float (&r)[G][4]) {
+  COPES_UNIT_COEFFS;
+  float L[G][4];
+  float L_min = 0.0f;  // L <= 0 for every word
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      x[i][e] = lattice_x(w[i][e]);
+      L[i][e] = lg2_approx(__fmaf_rn(-x[i][e], x[i][e], 1.0f));
+      L_min = fminf(L_min, L[i][e]);
+    }
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+      const unsigned long long Lp = pack_f32x2(L[i][2 * p], L[i][2 * p + 1]);
+      unsigned long long acc = splat_f32x2(unit_central[COPES_NORMAL_CENTRAL_DEGREE]);
+#pragma unroll
+      for (int k = COPES_NORMAL_CENTRAL_DEGREE - 1; k >= 0; --k) acc = fma_f32x2(acc, Lp, splat_f32x2(unit_central[k]));
+      unpack_f32x2(acc, r[i][2 * p], r[i][2 * p + 1]);
+    }
+  }
+  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
+#pragma unroll
+    for (int i = 0; i < G; ++i)
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (L[i][e] < COPES_NORMAL_L_SPLIT) r[i][e] = tail_ratio(unit_tail, L[i][e]);
+  }
+}
+
+// normal_parts_groups_x2 with every step on packed pairs (as normal_parts4_packed):
+// x2[i][p] = (x_2p, x_2p+1) and r2[i][p] = (r_2p, r_2p+1) of block i; the same values.
+template <int G>
+__device__ __forceinline__ void normal_parts_groups_packed(const uint32_t (&w)[G][4],
+                                                           unsigned long long (&x2)[G][2],
+                                                           unsigned long long (&r2)[G][2]) {
+  COPES_UNIT_COEFFS;
+  float L[G][4];
+  float L_min = 0.0f;
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+      const unsigned long long F = pack_f32x2(__uint_as_float((w[i][2 * p] & 0x007FFFFEu) | 0x40000001u),
+                                              __uint_as_float((w[i][2 * p + 1] & 0x007FFFFEu) | 0x40000001u));
+      x2[i][p] = add_f32x2(F, splat_f32x2(-3.0f));
+      float t0, t1;  // x^2 - 1 = -(1 - x^2)
+      unpack_f32x2(fma_f32x2(x2[i][p], x2[i][p], splat_f32x2(-1.0f)), t0, t1);
+      L[i][2 * p] = lg2_approx(-t0);
+      L[i][2 * p + 1] = lg2_approx(-t1);
+      L_min = fminf(L_min, fminf(L[i][2 * p], L[i][2 * p + 1]));
+      const unsigned long long Lp = pack_f32x2(L[i][2 * p], L[i][2 * p + 1]);
+      unsigned long long acc = splat_f32x2(unit_central[COPES_NORMAL_CENTRAL_DEGREE]);
+#pragma unroll
+      for (int k = COPES_NORMAL_CENTRAL_DEGREE - 1; k >= 0; --k) acc = fma_f32x2(acc, Lp, splat_f32x2(unit_central[k]));
+      r2[i][p] = acc;
+    }
+  }
+  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
+#pragma unroll
+    for (int i = 0; i < G; ++i)
+#pragma unroll
+      for (int p = 0; p < 2; ++p) {
+        float r0, r1;
+        unpack_f32x2(r2[i][p], r0, r1);
+        if (L[i][2 * p] < COPES_NORMAL_L_SPLIT) r0 = tail_ratio(unit_tail, L[i][2 * p]);
+        if (L[i][2 * p + 1] < COPES_NORMAL_L_SPLIT) r1 = tail_ratio(unit_tail, L[i][2 * p + 1]);
+        r2[i][p] = pack_f32x2(r0, r1);
+      }
+  }
+}
+
 // Two standard normals from two words (of different Philox blocks), their central
 // polynomials evaluated as one packed pair with compile-time coefficients and a single
 // warp vote for the tail: bit-identical to two normal_from_word calls.

@@ -74,6 +74,62 @@ __host__ __device__ __forceinline__ void philox4x32_10_rk(uint32_t c0, uint32_t 
   out[3] = c3;
 }
 
+// Philox4x32-10 at a counter (c0, 0, 0, tag) -- high word and aux zero -- with the work that
+// does not depend on c0 taken out.  With c1 = c2 = 0, round 0's second product is 0 and
+//   round 0: (c0, c1, c2, c3) <- (k0, 0, hi(M0 c0) ^ tag ^ k1, lo(M0 c0));
+//   round 1: M0 * k0 is a function of the key alone, so
+//            (c0, c1, c2, c3) <- (hi(M1 c2) ^ rk2, lo(M1 c2), hi(M0 k0) ^ lo(M0 c0) ^ rk3, lo(M0 k0));
+//   round 2: its c3 = lo(M0 k0) enters only word 2, XORed with rk5.
+// philox_folded_keys gathers those key-only terms with the remaining round keys:
+//   u = {k1 ^ tag, rk2, hi(M0 k0) ^ rk3, lo(M0 k0) ^ rk5, rk4, rk6, rk7, ..., rk19, 0};
+// philox4x32_10_folded then takes the counter's product M0 * c0 (which a caller computes
+// once for every key) and runs one multiply in round 1 and two in each of rounds 2..9:
+// 17 of the 20 32x32->64 multiplies, with the same output words as philox4x32_10.
+__host__ __device__ __forceinline__ void philox_folded_keys(const uint32_t rk[20], uint32_t tag, uint32_t u[20]) {
+  const uint64_t mk = (uint64_t)kPhiloxM0 * rk[0];
+  u[0] = rk[1] ^ tag;
+  u[1] = rk[2];
+  u[2] = (uint32_t)(mk >> 32) ^ rk[3];
+  u[3] = (uint32_t)mk ^ rk[5];
+  u[4] = rk[4];
+  for (int r = 3; r < 10; ++r) {
+    u[5 + 2 * (r - 3)] = rk[2 * r];
+    u[6 + 2 * (r - 3)] = rk[2 * r + 1];
+  }
+  u[19] = 0;
+}
+
+template <typename U>
+__host__ __device__ __forceinline__ void philox4x32_10_folded(uint32_t m0_lo, uint32_t m0_hi, const U &u,
+                                                              uint32_t out[4]) {
+  uint32_t c2 = m0_hi ^ u[0];  // after round 0
+  uint64_t p1 = (uint64_t)kPhiloxM1 * c2;
+  uint32_t c0 = (uint32_t)(p1 >> 32) ^ u[1];  // after round 1
+  uint32_t c1 = (uint32_t)p1;
+  c2 = u[2] ^ m0_lo;
+  uint64_t p0 = (uint64_t)kPhiloxM0 * c0;  // round 2
+  p1 = (uint64_t)kPhiloxM1 * c2;
+  c0 = (uint32_t)(p1 >> 32) ^ c1 ^ u[4];
+  c2 = (uint32_t)(p0 >> 32) ^ u[3];
+  c1 = (uint32_t)p1;
+  uint32_t c3 = (uint32_t)p0;
+#pragma unroll
+  for (int r = 3; r < 10; ++r) {
+    p0 = (uint64_t)kPhiloxM0 * c0;
+    p1 = (uint64_t)kPhiloxM1 * c2;
+    const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ u[5 + 2 * (r - 3)];
+    const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ u[6 + 2 * (r - 3)];
+    c1 = (uint32_t)p1;
+    c3 = (uint32_t)p0;
+    c0 = n0;
+    c2 = n2;
+  }
+  out[0] = c0;
+  out[1] = c1;
+  out[2] = c2;
+  out[3] = c3;
+}
+
 // Device error bits (set with atomicOr by a kernel that skipped an access).
 enum : unsigned {
   kErrTileRange = 1u,   // a tile outside [0, n_alloc) or longer than COPES_TILE_MAX

@@ -38,11 +38,14 @@ struct WStore<float> {
 
 // The update's prologue: folds the members into one weight per noise vector,
 //   w_j = sum_{i : noise(i) = j} sign_i f_i  (member order, fp32),
-// and expands each noise vector's Philox round keys into shared memory.
+// and expands each noise vector's Philox round keys into shared memory (and, when s_fk is
+// given, the folded keys of philox4x32_10_folded for the noise tag).
 __device__ __forceinline__ void noise_weights_to_smem(const UpdateArgs &a, float *s_w,
-                                                      uint32_t (*s_rk)[20]) {
+                                                      uint32_t (*s_rk)[20],
+                                                      uint32_t (*s_fk)[20] = nullptr) {
   for (int j = threadIdx.x; j < a.n_noise; j += blockDim.x) {
     philox_round_keys(a.seed_lo[j], a.seed_hi[j], s_rk[j]);
+    if (s_fk) philox_folded_keys(s_rk[j], COPES_TAG_NOISE, s_fk[j]);
     float acc = 0.0f;
     for (int m = a.noise_ptr[j]; m < a.noise_ptr[j + 1]; ++m) {
       const int i = a.noise_member[m];
