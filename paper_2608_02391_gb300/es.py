@@ -308,12 +308,14 @@ def gather_rewards(local: np.ndarray, n_members: int, group=None) -> np.ndarray:
 def population_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iteration: int,
                      cfg: ESConfig, d: int, evaluate: Callable[[int], float], group=None,
                      fitness_out: Optional[torch.Tensor] = None,
-                     partner: Optional[Partner] = None) -> torch.Tensor:
+                     partner: Optional[Partner] = None,
+                     rewards_out: Optional[np.ndarray] = None) -> torch.Tensor:
     """One ES iteration on subspace k, population-parallel over the ranks of `group`.
     Every rank holds the same theta; rank r evaluates members member_slice(r, R, N):
     perturb, evaluate(i) -> reward (host float) while the perturbation is live, and
     restores S afterwards.  The rewards are all-gathered, then every rank shapes the same
-    vector and applies the same fused update + commit, so the replicas stay identical."""
+    vector and applies the same fused update + commit, so the replicas stay identical.
+    rewards_out (host float32 [N]) receives the gathered rewards."""
     import torch.distributed as dist
     rank, world = dist.get_rank(group), dist.get_world_size(group)
     N = cfg.n_members
@@ -327,7 +329,10 @@ def population_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iter
 
     perturb_members(arena, sub, member_slice(rank, world, N), nid, sign, seeds, s_k, live, partner)
     copes.restore(arena, sub)
-    rewards = torch.from_numpy(gather_rewards(local, N, group)).to(arena.w.device)
+    gathered = gather_rewards(local, N, group)
+    if rewards_out is not None:
+        rewards_out[:] = gathered
+    rewards = torch.from_numpy(gathered).to(arena.w.device)
     f = fitness_out if fitness_out is not None else torch.empty_like(rewards)
     copes.shape_fitness(rewards, cfg.shaping, out=f)
     coef = copes.step_coef(cfg.alpha, N, s_k, cfg.convention)
@@ -337,21 +342,27 @@ def population_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iter
 
 # ------------------------------------------------------------------ checkpoint / resume
 def state_dict(arena: copes.Arena, cfg: ESConfig, next_iteration: int, **extra) -> dict:
-    """The resumable ES state: the fp32 master (host copy), the configuration and the next
-    iteration index.  Member seeds and noise are functions of (base seed, iteration,
-    subspace, member) and (seed, index), and partition seeds are part of `extra`, so
-    nothing else needs saving: a run resumed from this state continues bit for bit."""
+    """The resumable ES state: the fp32 master (host copy), the configuration, the next
+    iteration index and whether the arena keeps a second working copy w2.  Member seeds
+    and noise are functions of (base seed, iteration, subspace, member) and (seed, index),
+    and partition seeds are part of `extra`, so nothing else needs saving: a run resumed
+    from this state continues bit for bit.  The working copies are not saved: between ES
+    iterations both equal round(theta) and are rebuilt from the master."""
     return {"master": arena.master.detach().cpu().clone(), "working_dtype": str(arena.w.dtype),
-            "config": dict(cfg.__dict__), "next_iteration": int(next_iteration), **extra}
+            "second_copy": arena.w2 is not None, "config": dict(cfg.__dict__),
+            "next_iteration": int(next_iteration), **extra}
 
 
 def load_state(state: dict, device="cuda") -> tuple:
     """Rebuilds (arena, cfg, next_iteration) from state_dict's output: the master is
-    copied to the device and the working weights are committed from it (w = round(theta)
-    over the whole arena)."""
+    copied to the device and the working weights, with the second working copy when the
+    saved arena had one, are committed from it (w = w2 = round(theta) over the whole
+    arena)."""
     master = state["master"].to(device).contiguous()
     dtype = {"torch.bfloat16": torch.bfloat16, "torch.float32": torch.float32}[state["working_dtype"]]
-    arena = copes.Arena(torch.empty(master.numel(), dtype=dtype, device=device), master)
-    everything = copes.tiles_from_ranges([(0, master.numel())], device=device)
-    copes.context_commit(arena, everything)
+    n = master.numel()
+    w2 = torch.empty(n, dtype=dtype, device=device) if state.get("second_copy", False) else None
+    arena = copes.Arena(torch.empty(n, dtype=dtype, device=device), master, w2=w2)
+    everything = copes.tiles_from_ranges([(0, n)], device=device)
+    copes.context_commit(arena, everything)  # commit writes w2 too when it is set
     return arena, ESConfig(**state["config"]), state["next_iteration"]

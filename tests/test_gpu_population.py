@@ -1,12 +1,18 @@
 """Population-parallel ES on the GPU: two ranks (processes) with full replicas of theta
 split the members of every visit, exchange the reward scalars over gloo, and apply the
-same update.  After a cycle over the K subspaces their masters and working weights are
-bit-identical, and equal to a single process running the whole population.  The ranks'
-kernels never wait on one another: the only synchronisation is the host all-gather."""
+same update (Sec. 3.3: only seeds and scalar rewards travel).  On rank 0 the oracle
+recomputes every visit from the gathered rewards -- the shaped fitness, and the update of
+Eq. 13 on sampled elements of the subspace (its edges included) -- and the commit is
+checked bit for bit.  After a cycle over the K subspaces the ranks' masters and working
+weights are bit-identical, and equal to a single process running the whole population.
+The ranks' kernels never wait on one another: the only synchronisation is the host
+all-gather."""
+import datetime
 import hashlib
 import os
 import socket
 import sys
+import traceback
 
 import numpy as np
 import pytest
@@ -48,10 +54,34 @@ def _digest(torch, arena):
                           arena.w.view(torch.int16).cpu().numpy().tobytes()).hexdigest()
 
 
+def _oracle_check(torch, copes, arena, sub, k, cfg, rewards, f_gpu, idx, theta):
+    """The visit on subspace k against the oracle at the sampled indices idx (theta: the
+    master there before the visit)."""
+    sys.path.insert(0, os.path.join(ROOT, "tests"))
+    import oracle
+    from tolerances import assert_fitness_close, assert_update_close
+    N = cfg.n_members
+    f_ref = oracle.shape_fitness(rewards, oracle.SHAPE_ZSCORE)
+    assert_fitness_close(f_gpu, f_ref)
+    nid, sign, P = copes.member_table(N, cfg.pairing)
+    seeds = copes.member_seeds(cfg.base_seed, 0, k, P)
+    coef = np.float32(copes.step_coef(cfg.alpha, N, cfg.sigma, cfg.convention))
+    wj = oracle.noise_weights(nid, sign, f_ref, P)
+    _, exact, scale = oracle.update_at(idx.astype(np.uint64), theta, seeds, wj, coef)
+    it = torch.from_numpy(idx).cuda()
+    got = arena.master[it].cpu().numpy()
+    assert_update_close(got, exact, scale)
+    commit = oracle.bf16_bits_array(got)
+    for w in (arena.w, arena.w2):
+        if w is not None:
+            assert np.array_equal(w.view(torch.int16)[it].cpu().numpy().view(np.uint16), commit)
+
+
 def _worker(rank, world, port, out, dual):
     import torch.distributed as dist
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
-    dist.init_process_group("gloo", rank=rank, world_size=world)
+    # a bounded collective timeout: a rank that fails ends its peer's next all-gather
+    dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=120))
     try:
         torch, copes, es, arena, c, subs, cfg = _setup(dual)
         # dual: each rank evaluates its antithetic pairs on two working copies
@@ -60,8 +90,17 @@ def _worker(rank, world, port, out, dual):
         def evaluate(i):  # the reward of the live perturbation: a linear objective
             return float((c * arena.live.float()).sum().item())
 
+        rng = np.random.default_rng(7)
+        width = N_PARAMS // K
         for k in range(K):
-            es.population_visit(arena, subs[k], k, 0, cfg, N_PARAMS, evaluate, partner=partner)
+            lo, hi = k * width, (k + 1) * width  # subspace k of the contiguous split
+            idx = np.unique(np.concatenate([[lo, lo + 1, hi - 2, hi - 1], rng.integers(lo, hi, 3000)]))
+            theta = arena.master[torch.from_numpy(idx).cuda()].cpu().numpy()
+            rewards = np.zeros(N, np.float32)
+            f = es.population_visit(arena, subs[k], k, 0, cfg, N_PARAMS, evaluate, partner=partner,
+                                    rewards_out=rewards)
+            if rank == 0:
+                _oracle_check(torch, copes, arena, subs[k], k, cfg, rewards, f.cpu().numpy(), idx, theta)
         if dual:  # both copies hold the new context
             assert torch.equal(arena.w.view(torch.int16), arena.w2.view(torch.int16))
         copes.check()
@@ -77,23 +116,28 @@ def _worker(rank, world, port, out, dual):
                 es.round_robin_visit(arena1, subs1[k], k, 0, cfg1, N_PARAMS, rewards, evaluate=ev)
             copes.check()
             ref = _digest(torch, arena1)
-        out.put((rank, digest, ref))
+        out.put((rank, digest, ref, None))
+    except Exception:
+        out.put((rank, None, None, traceback.format_exc()))
     finally:
         dist.destroy_process_group()
 
 
 @pytest.mark.parametrize("dual", [False, True])
-def test_two_ranks_stay_bit_identical_and_match_one_process(dual):
+def test_two_ranks_match_the_oracle_and_one_process(dual):
     ctx = mp.get_context("spawn")
     out = ctx.Queue()
     port = _free_port()
     procs = [ctx.Process(target=_worker, args=(r, 2, port, out, dual)) for r in range(2)]
     for p in procs:
         p.start()
-    res = sorted(out.get(timeout=600) for _ in procs)
+    res = sorted((out.get(timeout=600) for _ in procs), key=lambda t: t[0])
     for p in procs:
         p.join(timeout=120)
+    errors = [e for *_, e in res if e]
+    assert not errors, "\n".join(errors)
+    for p in procs:
         assert p.exitcode == 0
-    (r0, d0, ref), (r1, d1, _) = res
+    (r0, d0, ref, _), (r1, d1, _, _) = res
     assert d0 == d1
     assert d0 == ref

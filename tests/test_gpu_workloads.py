@@ -382,6 +382,13 @@ def test_counters_beyond_2_34(copes):
     copes.perturb_pair(arena, sub, 77, 1e-3, buf, lo)
     assert torch.equal(arena.w[lo:hi].view(torch.int16), plus)
     assert torch.equal(buf.view(torch.int16), minus)
+    # ... and both members agree with the oracle on the sampled indices, on both sides of 2^34
+    theta = arena.master[torch.from_numpy(sample).cuda()].cpu().numpy()
+    g = sample.astype(np.uint64)
+    scale = np.maximum(np.abs(theta), np.abs(np.float32(1e-3) * oracle.noise(77, g)))
+    for s_sign, got in ((1.0, bf16_bits_of(arena.w, sample)), (-1.0, bf16_bits_of(buf, sample - lo))):
+        ref_bits, _ = oracle.perturb_at(g, theta, 77, s_sign * 1e-3, oracle.BF16)
+        assert_bf16_close(got, ref_bits.astype(np.uint16), scale)
     copes.check()
 
 
