@@ -323,6 +323,34 @@ def test_synchronous_composition_equals_sum_of_subspace_updates():
     assert np.array_equal(composed, (master.astype(np.float64) + delta).astype(np.float32))
 
 
+def test_synchronous_composed_update_rebuilt_with_numpy():
+    """Eq. 12 + Eq. 13 written out as linear algebra: joint z-scores over all K N_k rewards
+    (scipy), then theta+ = theta + sum_k (alpha / N_k) P_k E_k^T (s * f_k), with E_k the
+    member directions (antithetic: member 2j is +eps_j, 2j+1 is -eps_j) and P_k the
+    restriction to S_k (Eq. 8), each S_k's directions from its own seeds.  The oracle's
+    composed step lies within one fp32 ulp of that fp64 value."""
+    n, K, N_k, alpha = 1200, 3, 8, 5e-4
+    master = _rand_master(n, 12)
+    bounds = [0, 300, 700, n]  # unequal subspaces
+    r = np.random.default_rng(12).random(K * N_k).astype(np.float32)
+    f_all = oracle.shape_fitness(r, oracle.SHAPE_ZSCORE)
+    assert np.allclose(f_all, stats.zscore(r.astype(np.float64), ddof=0), rtol=1e-6, atol=1e-7)
+    nid, sign, P = oracle.member_table(N_k, oracle.ANTITHETIC)
+    th = master.copy()
+    ref = master.astype(np.float64)
+    for k in range(K):
+        lo, hi = bounds[k], bounds[k + 1]
+        seeds = _seeds(P, k=k)
+        f = f_all[k * N_k:(k + 1) * N_k]
+        c = np.float32(oracle.step_coef(alpha, N_k, 1e-3, oracle.COEF_PAPER))
+        oracle.update(th, oracle.make_subspace(ranges=[(lo, hi)]), nid, sign, f, seeds, c)
+        g = np.arange(lo, hi)
+        eps = np.stack([oracle.noise(int(s), g) for s in seeds])  # [P, d_k]
+        E = np.stack([(1.0 if i % 2 == 0 else -1.0) * eps[i // 2] for i in range(N_k)])  # [N_k, d_k]
+        ref[lo:hi] += np.float64(c) * (E.T @ f.astype(np.float64))
+    assert np.all(np.abs(th - ref) <= np.spacing(np.abs(ref).astype(np.float32)))
+
+
 def test_linear_objective_estimate_converges():
     """On r(theta) = c . theta with antithetic pairs, NONE shaping and coefficient
     alpha / (N sigma), the update divided by alpha is (1/P) sum_j (c . eps_j) eps_j, whose
