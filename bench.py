@@ -59,9 +59,12 @@ FALLBACK_HBM_GBS = 6800.0
 # ncu DRAM bytes per element of the dominant kernel (the pair perturb, or the plain perturb
 # under --weights single; bf16) from one capture each; a figure is dropped (traffic = null)
 # when the tile kernels' sources (source_sha) no longer match the hash it was taken on.
+# The pair perturb's figure comes from subspaces of 2^28 parameters, where the writes still
+# in L2 when the kernel ends are 2.4% of its traffic.
 NCU_TRAFFIC = {
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "35ede1dfa8ae5289",
-                     "bytes_per_elem": 7.225, "capture": "profiles/perturb_pair_4b_slice.md"},
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "a3e76802bf02a23c",
+                     "bytes_per_elem": 7.806, "capture": "profiles/perturb_pair_4b_slice.md",
+                     "case": "two 2^28-parameter subspaces (--case 4b-slice-big)"},
     "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "35ede1dfa8ae5289",
                 "bytes_per_elem": 5.413, "capture": "profiles/perturb_4b_slice.md"},
 }
@@ -542,6 +545,10 @@ def main():
     traffic = None
     if ncu["source_sha"] == source_sha() and ncu["bytes_per_elem"]:
         traffic = ncu["bytes_per_elem"] * mean_dk
+        traffic_note = (f"ncu dram__bytes_read + dram__bytes_write per element ({ncu['bytes_per_elem']} B) "
+                        f"on {ncu.get('case', 'a 2^26-parameter subspace')}, times this launch's elements")
+    else:
+        traffic_note = "no capture for the current kernel sources"
     props = torch.cuda.get_device_properties(local)
     clk = clocks.summary()
     n_normals_update = wl.n_members // 2
@@ -561,6 +568,7 @@ def main():
         "hbm_gbs": bytes_per_step * args.steps / (ms * 1e-3) / 1e9,
         "roofline": {"bound": "hbm", "kernel": "perturb_pair" if paired else "perturb", "achieved": achieved,
                      "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
+                     "traffic_source": traffic_note,
                      "peak_source": peak_src, "algorithmic_bytes_per_launch": perturb_bytes},
         "kernels": {
             ("perturb_pair" if paired else "perturb"): {
@@ -685,6 +693,11 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
     # writes), plus 8 B of index per member for lists
     lists = args.hash_mode in ("lists", "gathered")
     pb = ((8.0 if partner is not None else 6.0) + (8.0 if lists else 0.0)) * mean_dk
+    # the structural floor of a scattered pass: DRAM bytes per member it cannot avoid
+    n_w = (2 if partner is not None else 1)  # working-dtype arrays the perturb writes
+    floor_p = hash_sector_floor(wl.K, args.hash_mode, n_w)
+    floor_r = hash_sector_floor(wl.K, args.hash_mode, 2 if args.weights == "dual" else 1)
+    share = philox_block_share(torch, subs, wl.K, lists)
     value = job_throughput(world, d, args.steps, ms * 1e-3)
     out = {
         "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
@@ -703,10 +716,12 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
         "kernels": {
             ("perturb_pair" if partner is not None else "perturb"): {
                 "ms": per["perturb"], "launches": counts["perturb"], "GB/s": pb / (per["perturb"] * 1e-3) / 1e9,
-                "frac_hbm": pb / (per["perturb"] * 1e-3) / 1e9 / hbm},
+                "frac_hbm": pb / (per["perturb"] * 1e-3) / 1e9 / hbm,
+                **sector_floor_entry(floor_p, mean_dk, per["perturb"], hbm)},
             **({"perturb_partner": {"ms": per["partner"], "launches": counts["partner"]}}
                if "partner" in per else {}),
-            "restore": {"ms": per["restore"], "launches": counts["restore"]},
+            "restore": {"ms": per["restore"], "launches": counts["restore"],
+                        **sector_floor_entry(floor_r, mean_dk, per["restore"], hbm)},
             "update_fused_commit": {"ms": per["update"], "launches": counts["update"], "Tops": upd_tops,
                                     "frac_alu": upd_tops / alu_peak},
             "shape": {"ms": per["shape"], "launches": counts["shape"]},
@@ -717,7 +732,52 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
     }
     if "mask" in per:
         out["kernels"]["mask"] = {"ms": per["mask"], "launches": counts["mask"]}
+    out["philox_block_share"] = share
     print(json.dumps(out), flush=True)
+
+
+def hash_sector_floor(K: int, mode: str, n_w: int) -> dict:
+    """DRAM bytes per member that one pass over a hash subspace cannot avoid.  Members are
+    1 element in K, each element independently, and DRAM moves 64-byte sector pairs: a
+    pass that touches the members of an array of s-byte elements moves the pairs holding
+    at least one member, 64 (1 - (1 - 1/K)^(64/s)) bytes per 64/s elements, i.e.
+    64 (1 - (1 - 1/K)^(64/s)) / (64 / (s K)) bytes per member.  Index lists add their
+    8 contiguous bytes per member; a gathered master reads theta contiguously (4 bytes);
+    the replay mask adds its bits (K / 8 bytes per member).  n_w: working-dtype (bf16)
+    arrays written at the members (w, and w2 or the partner buffer)."""
+    q = 1.0 / K
+
+    def scattered(s):
+        m = 64 // s
+        return 64.0 * (1.0 - (1.0 - q) ** m) / (m * q)
+
+    parts = {"theta": 4.0 if mode == "gathered" else scattered(4), "w": n_w * scattered(2)}
+    if mode in ("lists", "gathered"):
+        parts["index"] = 8.0
+    if mode == "replay-mask":
+        parts["mask"] = K / 8.0
+    return {"bytes_per_member": sum(parts.values()), "parts": parts}
+
+
+def sector_floor_entry(floor: dict, members: float, ms: float, hbm: float) -> dict:
+    gbs = floor["bytes_per_member"] * members / (ms * 1e-3) / 1e9
+    return {"floor_bytes_per_member": floor["bytes_per_member"], "floor_GB/s": gbs, "frac_floor_hbm": gbs / hbm}
+
+
+def philox_block_share(torch, subs, K: int, lists: bool) -> dict:
+    """How often a hash subspace's consecutive members share a Philox block (the same
+    g >> 2), i.e. how many Philox calls per member a gather kernel could save by reusing
+    a block's words: measured on the index lists, or, for replayed subspaces, the
+    expectation for independent membership, (1/4) sum_{t=0..3} (1 - (1 - 1/K)^t)."""
+    if not lists:
+        v = sum(1.0 - (1.0 - 1.0 / K) ** t for t in range(4)) / 4.0
+        return {"value": v, "how": "expected for independent membership at this K"}
+    same, pairs = 0, 0
+    for sub in subs:
+        q = sub.tensor >> 2
+        same += int((q[1:] == q[:-1]).sum().item())
+        pairs += max(q.numel() - 1, 0)
+    return {"value": same / max(pairs, 1), "how": "measured on the index lists"}
 
 
 def host_link_gbs(torch, nbytes=1 << 30, reps=5):
