@@ -685,9 +685,13 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
     alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12
     P = wl.n_members // 2
     replay = args.hash_mode == "replay"  # the membership hash runs inside every kernel
-    # algorithmic work of one update launch: 28 lane-ops per normal, P normals per member;
-    # replay adds the membership hash of every element (one Philox call = 80 ops per 4)
-    upd_ops = 28.0 * P * mean_dk + (20.0 * d if replay else 0.0)
+    # algorithmic work of one update launch: a member's normal is one word of its own
+    # Philox call, so each (member, noise vector) costs a whole call (80 lane-ops) plus the
+    # uniform (3), transform (4) and update fma (1): 88 lane-ops per normal, P normals per
+    # member (a tile shares each call among 4 elements: 28).  Replay adds the membership
+    # hash of every element (one Philox call = 80 ops per 4 elements).
+    ops_per_normal = 88.0
+    upd_ops = ops_per_normal * P * mean_dk + (20.0 * d if replay else 0.0)
     upd_tops = upd_ops / (per["update"] * 1e-3) / 1e12
     # perturb: 6 B per member (read fp32, write bf16), 8 B for a pair perturb (two bf16
     # writes), plus 8 B of index per member for lists
@@ -723,7 +727,8 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
             "restore": {"ms": per["restore"], "launches": counts["restore"],
                         **sector_floor_entry(floor_r, mean_dk, per["restore"], hbm)},
             "update_fused_commit": {"ms": per["update"], "launches": counts["update"], "Tops": upd_tops,
-                                    "frac_alu": upd_tops / alu_peak},
+                                    "frac_alu": upd_tops / alu_peak, "ops_per_normal": ops_per_normal,
+                                    "normals_per_member": P},
             "shape": {"ms": per["shape"], "launches": counts["shape"]},
         },
         "clocks": clk,
