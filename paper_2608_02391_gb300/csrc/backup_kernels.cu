@@ -97,43 +97,18 @@ __global__ void __launch_bounds__(kThreads) backup_elem_kernel(const __grid_cons
   }
 }
 
-// The update: all P noise vectors regenerated per group in registers (j ascending), the
-// backup read only after the noise loop, the new context written to both copies.
-template <int G>
-__global__ void __launch_bounds__(kThreads) backup_update_kernel(const __grid_constant__ UpdateArgs a,
-                                                                 uint16_t *backup) {
-  __shared__ float s_w[COPES_MAX_NOISE];
-  __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
-  noise_weights_to_smem(a, s_w, s_rk);
-  uint64_t b, e;
-  if (!backup_tile(a.tiles, blockIdx.x, a.n_alloc, b, e)) return;
+// The update: all P noise vectors regenerated per group in registers (noise_sum_groups,
+// the tile update's loop), the backup read only after the noise loop, the new context
+// written to both copies.  Same launch shape as the tile update: G groups per thread,
+// 4 resident blocks per SM.
+template <int G, bool HI0>
+__device__ __forceinline__ void backup_update_tile(const UpdateArgs &a, uint16_t *backup, const float *s_w,
+                                                   const uint32_t (*s_rk)[20], const uint32_t (*s_fk)[20],
+                                                   uint64_t b, uint64_t e) {
   uint16_t *w = static_cast<uint16_t *>(a.w);
-  const int P = a.n_noise;
   for (uint64_t base = (b & ~3ull) + 4ull * threadIdx.x; base < e; base += 4ull * kThreads * G) {
     float acc[G][4];
-#pragma unroll
-    for (int i = 0; i < G; ++i)
-#pragma unroll
-      for (int k = 0; k < 4; ++k) acc[i][k] = 0.0f;
-    for (int j = 0; j < P; ++j) {
-      uint32_t rk[20];
-#pragma unroll
-      for (int r = 0; r < 20; r += 4) {
-        const uint4 v = *reinterpret_cast<const uint4 *>(&s_rk[j][r]);
-        rk[r] = v.x, rk[r + 1] = v.y, rk[r + 2] = v.z, rk[r + 3] = v.w;
-      }
-      const float wj = s_w[j];
-#pragma unroll
-      for (int i = 0; i < G; ++i) {
-        const uint64_t q = (base >> 2) + (uint64_t)kThreads * i;
-        uint32_t x[4];
-        philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, rk, x);
-        float eps[4];
-        normals4_x2(x, eps);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) acc[i][k] = __fmaf_rn(wj, eps[k], acc[i][k]);
-      }
-    }
+    noise_sum_groups<G, HI0>(base, a.n_noise, s_w, s_rk, s_fk, acc);
 #pragma unroll
     for (int i = 0; i < G; ++i) {
       const uint64_t g4 = base + 4ull * kThreads * i;
@@ -159,6 +134,21 @@ __global__ void __launch_bounds__(kThreads) backup_update_kernel(const __grid_co
   }
 }
 
+constexpr int kBackupUpdateGroups = 2;
+constexpr int kBackupUpdateBlocksPerSM = 4;
+
+__global__ void __launch_bounds__(kThreads, kBackupUpdateBlocksPerSM)
+    backup_update_kernel(const __grid_constant__ UpdateArgs a, uint16_t *backup) {
+  __shared__ float s_w[COPES_MAX_NOISE];
+  __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
+  __shared__ __align__(16) uint32_t s_fk[COPES_MAX_NOISE][20];
+  noise_weights_to_smem(a, s_w, s_rk, s_fk);
+  uint64_t b, e;
+  if (!backup_tile(a.tiles, blockIdx.x, a.n_alloc, b, e)) return;
+  if ((e >> 34) == 0) backup_update_tile<kBackupUpdateGroups, true>(a, backup, s_w, s_rk, s_fk, b, e);
+  else backup_update_tile<kBackupUpdateGroups, false>(a, backup, s_w, s_rk, s_fk, b, e);
+}
+
 cudaError_t launch_backup_elementwise(int op, const ElemArgs &a, uint16_t *backup, cudaStream_t s) {
   if (a.n_tiles == 0) return cudaSuccess;
   const unsigned grid = (unsigned)a.n_tiles;
@@ -173,7 +163,7 @@ cudaError_t launch_backup_elementwise(int op, const ElemArgs &a, uint16_t *backu
 
 cudaError_t launch_backup_update(const UpdateArgs &a, uint16_t *backup, cudaStream_t s) {
   if (a.n_tiles == 0) return cudaSuccess;
-  backup_update_kernel<4><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a, backup);
+  backup_update_kernel<<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a, backup);
   return cudaGetLastError();
 }
 

@@ -121,23 +121,6 @@ __device__ __forceinline__ float normal_from_word(uint32_t w) {
   return __fmul_rn(x, r);
 }
 
-// eps for the four words of one Philox block, the central polynomial on packed fp32
-// pairs with compile-time (c, c) coefficients: bit-identical to four normal_from_word
-// calls, at fewer issue slots and without coefficient registers.
-__device__ __forceinline__ void normals4_x2(const uint32_t (&w)[4], float (&eps)[4]) {
-  COPES_UNIT_COEFFS;
-  unsigned long long c2[COPES_NORMAL_CENTRAL_DEGREE + 1];
-#pragma unroll
-  for (int k = 0; k <= COPES_NORMAL_CENTRAL_DEGREE; ++k) {
-    const unsigned long long b = __float_as_uint(unit_central[k]);
-    c2[k] = (b << 32) | b;
-  }
-  float x[4], r[4];
-  normal_parts4_x2(w, c2, unit_tail, x, r);
-#pragma unroll
-  for (int e = 0; e < 4; ++e) eps[e] = __fmul_rn(x[e], r[e]);
-}
-
 __device__ __forceinline__ unsigned long long add_f32x2(unsigned long long a, unsigned long long b) {
   unsigned long long d;
   asm("add.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
@@ -153,97 +136,12 @@ __device__ __forceinline__ unsigned long long splat_f32x2(float c) {
   return (b << 32) | b;
 }
 
-// normal_parts4_x2 with every step on packed pairs: x2[p] = (x_2p, x_2p+1) and
-// r2[p] = (r_2p, r_2p+1).  Each packed op rounds like its scalar form, and x^2 - 1 is the
-// exact negative of 1 - x^2 under round-to-nearest, so the results are those of
-// normal_parts4_x2 bit for bit, at fewer issue slots.
-template <int NC, int NT>
-__device__ __forceinline__ void normal_parts4_packed(const uint32_t (&w)[4],
-                                                     const unsigned long long (&central2)[NC],
-                                                     const float (&tail)[NT],
-                                                     unsigned long long (&x2)[2],
-                                                     unsigned long long (&r2)[2]) {
-  float L[4];
-#pragma unroll
-  for (int p = 0; p < 2; ++p) {
-    const unsigned long long F = pack_f32x2(__uint_as_float((w[2 * p] & 0x007FFFFEu) | 0x40000001u),
-                                            __uint_as_float((w[2 * p + 1] & 0x007FFFFEu) | 0x40000001u));
-    x2[p] = add_f32x2(F, splat_f32x2(-3.0f));
-    float t0, t1;  // x^2 - 1 = -(1 - x^2)
-    unpack_f32x2(fma_f32x2(x2[p], x2[p], splat_f32x2(-1.0f)), t0, t1);
-    L[2 * p] = lg2_approx(-t0);
-    L[2 * p + 1] = lg2_approx(-t1);
-    const unsigned long long Lp = pack_f32x2(L[2 * p], L[2 * p + 1]);
-    unsigned long long acc = central2[NC - 1];
-#pragma unroll
-    for (int i = NC - 2; i >= 0; --i) acc = fma_f32x2(acc, Lp, central2[i]);
-    r2[p] = acc;
-  }
-  const float L_min = fminf(fminf(L[0], L[1]), fminf(L[2], L[3]));
-  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
-#pragma unroll
-    for (int p = 0; p < 2; ++p) {
-      float r0, r1;
-      unpack_f32x2(r2[p], r0, r1);
-      if (L[2 * p] < COPES_NORMAL_L_SPLIT) r0 = tail_ratio(tail, L[2 * p]);
-      if (L[2 * p + 1] < COPES_NORMAL_L_SPLIT) r1 = tail_ratio(tail, L[2 * p + 1]);
-      r2[p] = pack_f32x2(r0, r1);
-    }
-  }
-}
-
-// eps for the four words of one Philox block as two packed pairs, with compile-time
-// coefficients: bit-identical to normals4_x2.
-__device__ __forceinline__ void normals4_packed(const uint32_t (&w)[4], unsigned long long (&eps2)[2]) {
-  COPES_UNIT_COEFFS;
-  unsigned long long c2[COPES_NORMAL_CENTRAL_DEGREE + 1];
-#pragma unroll
-  for (int k = 0; k <= COPES_NORMAL_CENTRAL_DEGREE; ++k) c2[k] = splat_f32x2(unit_central[k]);
-  unsigned long long x2[2], r2[2];
-  normal_parts4_packed(w, c2, unit_tail, x2, r2);
-#pragma unroll
-  for (int p = 0; p < 2; ++p) eps2[p] = mul_f32x2(x2[p], r2[p]);
-}
-
-// The normals of G Philox blocks with a single warp vote for the tail: every block's central
-// polynomial on packed pairs with compile-time coefficients, then, only when some lane of
-// the warp holds a word in the tail, the tail polynomial for those words.  Each result is
-// the same function of its word as in normals4_x2, so the outputs equal G calls of it bit
-// for bit, with one vote instead of G.  eps = x * r.
-template <int G>
-__device__ __forceinline__ void normal_parts_groups_x2(const uint32_t (&w)[G][4], float (&x)[G][4],
-                                                       float (&r)[G][4]) {
-  COPES_UNIT_COEFFS;
-  float L[G][4];
-  float L_min = 0.0f;  // L <= 0 for every word
-#pragma unroll
-  for (int i = 0; i < G; ++i) {
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      x[i][e] = lattice_x(w[i][e]);
-      L[i][e] = lg2_approx(__fmaf_rn(-x[i][e], x[i][e], 1.0f));
-      L_min = fminf(L_min, L[i][e]);
-    }
-#pragma unroll
-    for (int p = 0; p < 2; ++p) {
-      const unsigned long long Lp = pack_f32x2(L[i][2 * p], L[i][2 * p + 1]);
-      unsigned long long acc = splat_f32x2(unit_central[COPES_NORMAL_CENTRAL_DEGREE]);
-#pragma unroll
-      for (int k = COPES_NORMAL_CENTRAL_DEGREE - 1; k >= 0; --k) acc = fma_f32x2(acc, Lp, splat_f32x2(unit_central[k]));
-      unpack_f32x2(acc, r[i][2 * p], r[i][2 * p + 1]);
-    }
-  }
-  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
-#pragma unroll
-    for (int i = 0; i < G; ++i)
-#pragma unroll
-      for (int e = 0; e < 4; ++e)
-        if (L[i][e] < COPES_NORMAL_L_SPLIT) r[i][e] = tail_ratio(unit_tail, L[i][e]);
-  }
-}
-
-// normal_parts_groups_x2 with every step on packed pairs (as normal_parts4_packed):
-// x2[i][p] = (x_2p, x_2p+1) and r2[i][p] = (r_2p, r_2p+1) of block i; the same values.
+// The normals of G Philox blocks with a single warp vote for the tail, every step on packed
+// fp32 pairs with compile-time coefficients: each block's central polynomial, then, only
+// when some lane of the warp holds a word in the tail, the tail polynomial for those words.  x2[i][p] = (x_2p, x_2p+1) and r2[i][p] = (r_2p, r_2p+1) of
+// block i, eps = x * r.  Each packed op rounds like its scalar form and x^2 - 1 is the
+// exact negative of 1 - x^2 under round-to-nearest, so each eps is normal_from_word of its
+// word bit for bit, with one vote for G blocks instead of one per word.
 template <int G>
 __device__ __forceinline__ void normal_parts_groups_packed(const uint32_t (&w)[G][4],
                                                            unsigned long long (&x2)[G][2],

@@ -353,80 +353,18 @@ cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, c
 // ------------------------------------------------------------------------- update
 // One block per tile: the prologue (noise_weights_to_smem) folds the members into one
 // weight per noise vector; every thread then regenerates all P noise vectors for its G
-// groups in registers and accumulates acc = sum_j w_j eps_j (j ascending),
-// theta = fma(coef, acc, theta).  Per noise vector a thread runs the G groups' Philox calls
-// first, then their transforms with one tail vote (normal_parts_groups_*), then the
-// accumulation.  HI0 (every counter below 2^32): Philox in the folded form, with each
-// group's product M0 * q computed once for all noise vectors.
-// PACK: the transform's steps and the accumulation on packed fp32 pairs (the same values).
-template <typename WT, int G, bool COMMIT, bool HI0, bool PACK>
+// groups in registers (noise_sum_groups), acc = sum_j w_j eps_j (j ascending), and
+// writes theta = fma(coef, acc, theta) and, with COMMIT, its rounding to the working
+// copies.
+template <typename WT, int G, bool COMMIT, bool HI0>
 __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_w,
                                             const uint32_t (*s_rk)[20], const uint32_t (*s_fk)[20],
                                             uint64_t b, uint64_t e) {
   float *__restrict__ master = a.master;
   const uint64_t lo = b & ~3ull;
-  const int P = a.n_noise;
   for (uint64_t base = lo + 4ull * threadIdx.x; base < e; base += 4ull * kThreads * G) {
     float acc[G][4];
-    unsigned long long acc2[G][2];  // PACK: the accumulators as pairs (acc[i][2p], acc[i][2p+1])
-#pragma unroll
-    for (int i = 0; i < G; ++i) {
-      acc2[i][0] = acc2[i][1] = 0ull;
-#pragma unroll
-      for (int k = 0; k < 4; ++k) acc[i][k] = 0.0f;
-    }
-    const uint32_t q_lo = (uint32_t)(base >> 2);  // counter of group 0 (HI0: the whole counter)
-    uint32_t m0_lo[G], m0_hi[G];                  // HI0: M0 * counter of each group
-    if (HI0) {
-#pragma unroll
-      for (int i = 0; i < G; ++i) {
-        const uint64_t m = (uint64_t)kPhiloxM0 * (q_lo + kThreads * i);
-        m0_lo[i] = (uint32_t)m;
-        m0_hi[i] = (uint32_t)(m >> 32);
-      }
-    }
-    for (int j = 0; j < P; ++j) {
-      uint32_t k[20];
-      const uint32_t *src = HI0 ? s_fk[j] : s_rk[j];
-#pragma unroll
-      for (int r = 0; r < 20; r += 4) {
-        const uint4 v = *reinterpret_cast<const uint4 *>(src + r);
-        k[r] = v.x, k[r + 1] = v.y, k[r + 2] = v.z, k[r + 3] = v.w;
-      }
-      const float wj = s_w[j];
-      uint32_t w[G][4];
-#pragma unroll
-      for (int i = 0; i < G; ++i) {
-        if (HI0) {
-          philox4x32_10_folded(m0_lo[i], m0_hi[i], k, w[i]);
-        } else {
-          const uint64_t q = (base >> 2) + kThreads * i;
-          philox4x32_10_rk((uint32_t)q, (uint32_t)(q >> 32), 0u, COPES_TAG_NOISE, k, w[i]);
-        }
-      }
-      if constexpr (PACK) {
-        unsigned long long x2[G][2], r2[G][2];
-        normal_parts_groups_packed<G>(w, x2, r2);
-#pragma unroll
-        for (int i = 0; i < G; ++i)
-#pragma unroll
-          for (int p = 0; p < 2; ++p) acc2[i][p] = fma_f32x2(splat_f32x2(wj), mul_f32x2(x2[i][p], r2[i][p]), acc2[i][p]);
-      } else {
-        float x[G][4], r[G][4];
-        normal_parts_groups_x2<G>(w, x, r);
-#pragma unroll
-        for (int i = 0; i < G; ++i)
-#pragma unroll
-          for (int q = 0; q < 4; ++q) acc[i][q] = __fmaf_rn(wj, __fmul_rn(x[i][q], r[i][q]), acc[i][q]);
-      }
-    }
-    if constexpr (PACK) {
-#pragma unroll
-      for (int i = 0; i < G; ++i) {
-        unpack_f32x2(acc2[i][0], acc[i][0], acc[i][1]);
-        unpack_f32x2(acc2[i][1], acc[i][2], acc[i][3]);
-      }
-    }
+    noise_sum_groups<G, HI0>(base, a.n_noise, s_w, s_rk, s_fk, acc);
     // theta is read only now, after the noise loop, so it occupies no registers there
 #pragma unroll
     for (int i = 0; i < G; ++i) {
@@ -459,20 +397,14 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
   }
 }
 
-// Launch shapes of the tile update, by the number of noise vectors P: groups per thread and
-// resident blocks per SM (registers: 65536 / (256 x blocks) a thread).  With few noise
-// vectors (P <= kFewNoise) the master traffic weighs more and the transform runs on packed
-// pairs throughout.
+// Launch shape of the tile update: groups per thread and resident blocks per SM
+// (registers: 65536 / (256 x blocks) a thread).  Measured best for P = 4, 16 and 64.
 constexpr int kUpdateGroups = 2;
 constexpr int kUpdateBlocksPerSM = 4;
-constexpr int kUpdateGroupsFewNoise = 2;
-constexpr int kUpdateBlocksPerSMFewNoise = 4;
-constexpr bool kUpdatePackFewNoise = true;
-constexpr int kFewNoise = 8;
 
 // One block per tile; the prologue folds the members into noise weights and expands each
 // noise vector's Philox keys (round keys, and the folded form) into shared memory.
-template <typename WT, int G, bool COMMIT, int BLOCKS, bool PACK>
+template <typename WT, int G, bool COMMIT, int BLOCKS>
 __global__ void __launch_bounds__(kThreads, BLOCKS) update_tiles_kernel(const __grid_constant__ UpdateArgs a) {
   __shared__ float s_w[COPES_MAX_NOISE];
   __shared__ __align__(16) uint32_t s_rk[COPES_MAX_NOISE][20];
@@ -484,8 +416,8 @@ __global__ void __launch_bounds__(kThreads, BLOCKS) update_tiles_kernel(const __
     if (threadIdx.x == 0) flag_error(kErrTileRange);
     return;
   }
-  if ((e >> 34) == 0) update_tile<WT, G, COMMIT, true, PACK>(a, s_w, s_rk, s_fk, b, e);
-  else update_tile<WT, G, COMMIT, false, PACK>(a, s_w, s_rk, s_fk, b, e);
+  if ((e >> 34) == 0) update_tile<WT, G, COMMIT, true>(a, s_w, s_rk, s_fk, b, e);
+  else update_tile<WT, G, COMMIT, false>(a, s_w, s_rk, s_fk, b, e);
 }
 
 // Gather form of the update: indices staged through shared memory as in
@@ -564,11 +496,7 @@ template <typename WT, bool COMMIT>
 static cudaError_t launch_update_typed(int kind, const UpdateArgs &a, cudaStream_t s) {
   if (kind == COPES_SUBSPACE_TILES) {
     if (a.n_tiles == 0) return cudaSuccess;
-    if (a.n_noise <= kFewNoise)
-      update_tiles_kernel<WT, kUpdateGroupsFewNoise, COMMIT, kUpdateBlocksPerSMFewNoise, kUpdatePackFewNoise>
-          <<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
-    else
-      update_tiles_kernel<WT, kUpdateGroups, COMMIT, kUpdateBlocksPerSM, false><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+    update_tiles_kernel<WT, kUpdateGroups, COMMIT, kUpdateBlocksPerSM><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
   } else {
     if (a.n_index == 0) return cudaSuccess;
     const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;

@@ -133,7 +133,7 @@ def run_update(copes, arena, sub, rewards, pairing, mode, seeds_base, coef, fuse
 
 @pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
 @pytest.mark.parametrize("kind,tile", [("tiles", 4096), ("tiles", 777), ("indices", 0)])
-@pytest.mark.parametrize("n_members,pairing", [(8, 1), (32, 1), (128, 1), (5, 0), (256, 0)])
+@pytest.mark.parametrize("n_members,pairing", [(2, 1), (3, 0), (8, 1), (32, 1), (128, 1), (5, 0), (256, 0)])
 def test_update_parity(copes, dtype, kind, tile, n_members, pairing):
     theta = theta_np(seed=n_members)
     arena = make(copes, dtype, theta)

@@ -57,6 +57,21 @@ def test_static_scratch_matches_workspace_version_twice(copes, K, seed):
     copes.check()
 
 
+def test_static_scratch_lists_match_the_oracle(copes):
+    """The static entry point's lists against the oracle's hash partition (Eq. 7: element
+    e of tensor tid goes to subspace floor(x K / 2^32), x its partition Philox word),
+    on a fresh scratch state and after another partition reused it."""
+    import oracle
+    layout = copes.Layout(NUMEL, TENSOR_IDS)
+    for K, seed in ((3, 21), (8, 1088)):
+        subs = copes.hash_partition_static(layout, K, seed)
+        torch.cuda.synchronize()
+        for k in range(K):
+            ref = oracle.hash_list(NUMEL, TENSOR_IDS, K, seed, k)
+            assert np.array_equal(subs[k].tensor.cpu().numpy(), ref), (K, k)
+    copes.check()
+
+
 def test_static_scratch_rejects_oversize_and_short_lists(copes):
     big = copes.Layout([1 << 31, 1 << 31])  # needs far more than the fixed scratch
     rc, _ = _static_call(copes, big, 16, 1)
