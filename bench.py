@@ -62,7 +62,7 @@ FALLBACK_HBM_GBS = 6800.0
 # The pair perturb's figure comes from subspaces of 2^28 parameters, where the writes still
 # in L2 when the kernel ends are 2.4% of its traffic.
 NCU_TRAFFIC = {
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "a3e76802bf02a23c",
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "0a229ad5a5b0a07d",
                      "bytes_per_elem": 7.806, "capture": "profiles/perturb_pair_4b_slice.md",
                      "case": "two 2^28-parameter subspaces (--case 4b-slice-big)"},
     "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "35ede1dfa8ae5289",
