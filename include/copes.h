@@ -89,6 +89,9 @@ typedef struct {
   int dtype;        /* COPES_BF16 or COPES_FP32 (the dtype of w)                       */
   void *w2;         /* device, optional: second working buffer (16-byte aligned), or NULL */
 } copes_params;
+/* w, master and w2 must be pairwise disjoint byte ranges (n_alloc elements each): the
+ * kernels read the master while they write the working buffers.  Every call that takes
+ * copes_params checks this and returns COPES_ERR_INVALID_ARG otherwise. */
 
 /* A subspace S (Eq. 7 / Eq. 8: the support of P_k).
  *  TILES:       a device array of n_tiles [begin, end) pairs of uint64 global indices
@@ -322,8 +325,8 @@ int copes_perturb(const copes_params *p, const copes_subspace *S, uint64_t seed,
  * of the noise.  partner: caller-owned device buffer of the working dtype (2 B per element
  * for bf16, 4 B for fp32), 16-byte aligned, holding global indices
  * [partner_base, partner_base + partner_len) at offsets 0 .. partner_len - 1; partner_base
- * is a multiple of 4, the range lies inside the arena and the buffer does not overlap w
- * (COPES_ERR_ALIGNMENT / COPES_ERR_SIZE / COPES_ERR_INVALID_ARG otherwise).  It may be the
+ * is a multiple of 4, the range lies inside the arena and the buffer overlaps neither w
+ * nor the master (COPES_ERR_ALIGNMENT / COPES_ERR_SIZE / COPES_ERR_INVALID_ARG otherwise).  It may be the
  * arena's second working buffer w2.  An element of S outside that range is skipped and reported
  * by copes_check (bit 16).  Entries of the buffer outside S are untouched. */
 int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t seed,
