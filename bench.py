@@ -60,10 +60,10 @@ FALLBACK_HBM_GBS = 6800.0
 # under --weights single; bf16) from one capture each; a figure is dropped (traffic = null)
 # when the tile kernels' sources (source_sha) no longer match the hash it was taken on.
 # The pair perturb's figure comes from subspaces of 2^28 parameters, where the writes still
-# in L2 when the kernel ends are 2.4% of its traffic.
+# in L2 when the kernel ends are about 2% of its traffic.
 NCU_TRAFFIC = {
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "0a229ad5a5b0a07d",
-                     "bytes_per_elem": 7.806, "capture": "profiles/perturb_pair_4b_slice.md",
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "e98acb47d0b938ec",
+                     "bytes_per_elem": 7.827, "capture": "profiles/perturb_pair_4b_slice.md",
                      "case": "two 2^28-parameter subspaces (--case 4b-slice-big)"},
     "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "35ede1dfa8ae5289",
                 "bytes_per_elem": 5.413, "capture": "profiles/perturb_4b_slice.md"},

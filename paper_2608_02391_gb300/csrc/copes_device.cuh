@@ -182,6 +182,44 @@ __device__ __forceinline__ void normal_parts_groups_packed(const uint32_t (&w)[G
   }
 }
 
+// normal_parts4_x2 over G Philox blocks with a single warp vote for the tail: every
+// block's x and r = R(L) scaled by the caller's coefficients (central2 as (c, c) pairs),
+// then, only when some lane of the warp holds a word in the tail, the tail polynomial for
+// those words.  Each result is the same function of its word as in normal_parts4_x2, bit
+// for bit, with one vote for G blocks instead of one per block.
+template <int G, int NC, int NT>
+__device__ __forceinline__ void normal_parts_groups_x2(const uint32_t (&w)[G][4],
+                                                       const unsigned long long (&central2)[NC],
+                                                       const float (&tail)[NT], float (&x)[G][4],
+                                                       float (&r)[G][4]) {
+  float L[G][4];
+  float L_min = 0.0f;  // L <= 0 for every word
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      x[i][e] = lattice_x(w[i][e]);
+      L[i][e] = lg2_approx(__fmaf_rn(-x[i][e], x[i][e], 1.0f));
+      L_min = fminf(L_min, L[i][e]);
+    }
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+      const unsigned long long Lp = pack_f32x2(L[i][2 * p], L[i][2 * p + 1]);
+      unsigned long long acc = central2[NC - 1];
+#pragma unroll
+      for (int k = NC - 2; k >= 0; --k) acc = fma_f32x2(acc, Lp, central2[k]);
+      unpack_f32x2(acc, r[i][2 * p], r[i][2 * p + 1]);
+    }
+  }
+  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
+#pragma unroll
+    for (int i = 0; i < G; ++i)
+#pragma unroll
+      for (int e = 0; e < 4; ++e)
+        if (L[i][e] < COPES_NORMAL_L_SPLIT) r[i][e] = tail_ratio(tail, L[i][e]);
+  }
+}
+
 // Two standard normals from two words (of different Philox blocks), their central
 // polynomials evaluated as one packed pair with compile-time coefficients and a single
 // warp vote for the tail: bit-identical to two normal_from_word calls.

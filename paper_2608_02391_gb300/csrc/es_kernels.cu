@@ -60,11 +60,41 @@ __device__ __forceinline__ void elem_values(const ElemArgs &a, uint32_t q_lo, ui
   }
 }
 
+// One step of the pair perturb over the thread's G groups of an aligned tile whose
+// counters are all below 2^32: the G groups' Philox calls first, then their transforms
+// with one tail vote (normal_parts_groups_x2), then each group's two members -- the
+// values elem_values<kOpPerturbPair> computes, bit for bit.  Groups past the tile's end
+// are generated but not stored.
+template <typename WT, int G>
+__device__ __forceinline__ void pair_perturb_step(const ElemArgs &a, uint64_t b, uint32_t len, uint32_t off,
+                                                  uint32_t q0_lo, const float (&th)[G][4]) {
+  uint32_t w[G][4];
+#pragma unroll
+  for (int i = 0; i < G; ++i)
+    philox4x32_10_rk(q0_lo + ((off + 4u * kThreads * i) >> 2), 0u, 0u, COPES_TAG_NOISE, a.rk, w[i]);
+  float x[G][4], r[G][4];  // r = a * R(L)
+  normal_parts_groups_x2<G>(w, a.coeffs.central2, a.coeffs.tail, x, r);
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+    const uint32_t o = off + 4u * kThreads * i;
+    if (o >= len) continue;
+    float v[4], vp[4];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      v[e] = __fmaf_rn(r[i][e], x[i][e], th[i][e]);
+      vp[e] = __fmaf_rn(-r[i][e], x[i][e], th[i][e]);
+    }
+    WStore<WT>::full(a.w, b + o, v);
+    WStore<WT>::full(a.partner, b + o - a.partner_base, vp);
+  }
+}
+
 // Tile whose ends are multiples of 4: every group is whole.  Tile-local pointers and
 // 32-bit offsets; G groups per thread per step, loads issued before the math.
 // HI0: every counter of the tile is below 2^32 (its high word is the constant 0), so the
 // counter arithmetic stays in 32 bits and the compiler drops Philox's first-round
-// multiply of word 2 and hoists the second round's multiply of word 0.
+// multiply of word 2 and hoists the second round's multiply of word 0; the pair perturb
+// then takes the G groups together (pair_perturb_step).
 template <int OP, typename WT, int G, bool HI0>
 __device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b, uint32_t len) {
   float *__restrict__ mt = a.master + b;
@@ -82,6 +112,10 @@ __device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b,
 #pragma unroll
         for (int k = 0; k < 4; ++k) th[i][k] = 0.0f;
       }
+    }
+    if constexpr (OP == kOpPerturbPair && HI0) {
+      pair_perturb_step<WT, G>(a, b, len, off, q0_lo, th);
+      continue;
     }
 #pragma unroll
     for (int i = 0; i < G; ++i) {
@@ -155,9 +189,15 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
   }
 }
 
-// One block per tile [tiles[2t], tiles[2t+1]).  3 resident blocks per SM leave 85 registers a
-// thread for G = 8 groups in flight (measured 2% faster than G = 4 at 4 blocks, the next best).
-constexpr int kElemBlocksPerSM = 3;
+// One block per tile [tiles[2t], tiles[2t+1]).  Launch shapes, measured on the 4B set:
+// the pair perturb takes G = 4 groups per step together (one tail vote for the four) at 4
+// resident blocks per SM (64 registers a thread): 0.603 ms against 0.631 ms for G = 8 one
+// group at a time at 3 blocks.  The other ops take G = 8 groups one at a time at 3 blocks
+// per SM (85 registers), which the plain perturb runs faster (0.532 against 0.544 ms).
+template <int OP>
+constexpr int elem_blocks_per_sm() { return OP == kOpPerturbPair ? 4 : 3; }
+template <int OP>
+constexpr int elem_groups() { return OP == kOpPerturbPair ? 4 : 8; }
 
 // A tile outside [partner_base, partner_base + partner_len) is skipped and flagged.
 __device__ __forceinline__ bool partner_covers(const ElemArgs &a, uint64_t b, uint64_t e) {
@@ -165,7 +205,7 @@ __device__ __forceinline__ bool partner_covers(const ElemArgs &a, uint64_t b, ui
 }
 
 template <int OP, typename WT, int G>
-__global__ void __launch_bounds__(kThreads, kElemBlocksPerSM) elem_tiles_kernel(const ElemArgs a) {
+__global__ void __launch_bounds__(kThreads, elem_blocks_per_sm<OP>()) elem_tiles_kernel(const ElemArgs a) {
   const uint64_t t = blockIdx.x;
   const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
   if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
@@ -318,7 +358,7 @@ static cudaError_t launch_elem_typed(int kind, const ElemArgs &a, cudaStream_t s
     elem_index_kernel<OP, WT, true><<<(unsigned)blocks, kThreads, 0, s>>>(a);
   } else if (kind == COPES_SUBSPACE_TILES) {
     if (a.n_tiles == 0) return cudaSuccess;
-    constexpr int G = 8;
+    constexpr int G = elem_groups<OP>();
     if constexpr (OP == kOpPartner)
       partner_tiles_kernel<WT, G><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
     else
