@@ -221,17 +221,36 @@ int split_tiles(const Ranges &r, uint64_t tile_size, std::vector<uint64_t> &tile
   return COPES_OK;
 }
 
+// Writes the tile table of r on `stream`.  Up to kTileRangesMax ranges, a kernel expands
+// them on the device from its launch parameters: no host copy of the table, which from
+// pageable memory can make the host wait for the stream.  Longer range lists (random
+// chunks) are split on the host and copied.
 int emit_tiles(const Ranges &r, uint64_t tile_size, uint64_t *tiles, uint64_t capacity,
                uint64_t *count, cudaStream_t s, const char *who) {
-  std::vector<uint64_t> host;
-  split_tiles(r, tile_size, host);
-  const uint64_t n = host.size() / 2;
+  uint64_t n = 0;
+  for (const auto &x : r) n += (x.second - x.first + tile_size - 1) / tile_size;
   *count = n;
   if (!tiles) return COPES_OK;
   if (capacity < n) return fail(COPES_ERR_WORKSPACE, "%s: %llu tiles needed, capacity %llu", who,
                                 (unsigned long long)n, (unsigned long long)capacity);
   if (!aligned(tiles, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: tiles must be 16-byte aligned", who);
   if (n == 0) return COPES_OK;
+  if (r.size() <= (size_t)copes::kTileRangesMax) {
+    static thread_local copes::TileRanges tr;  // 24 KB: kept off the stack
+    tr.n_ranges = (int)r.size();
+    tr.tile_size = tile_size;
+    uint64_t first = 0;
+    for (size_t i = 0; i < r.size(); ++i) {
+      tr.begin[i] = r[i].first;
+      tr.end[i] = r[i].second;
+      tr.first[i] = first;
+      first += (r[i].second - r[i].first + tile_size - 1) / tile_size;
+    }
+    tr.first[r.size()] = first;
+    return launch_status(copes::launch_tile_expand(tr, tiles, s), who);
+  }
+  std::vector<uint64_t> host;
+  split_tiles(r, tile_size, host);
   // Pageable source: the call returns once the data is staged, so `host` may go away.
   return launch_status(cudaMemcpyAsync(tiles, host.data(), n * 16, cudaMemcpyHostToDevice, s), who);
 }

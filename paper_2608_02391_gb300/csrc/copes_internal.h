@@ -238,6 +238,17 @@ cudaError_t launch_hash_scan(const uint32_t *hist, uint64_t n_htiles, int K, uin
 cudaError_t launch_hash_scatter(const HashTensor *tensors, int n_tensors, uint64_t n_htiles,
                                 int K, uint64_t seed, const uint64_t *offsets,
                                 int64_t *const *lists, cudaStream_t s);
+// A tile table's ranges as launch parameters: range r covers [begin[r], end[r]) and its
+// tiles start at index first[r]; first[n_ranges] is the tile count.
+constexpr int kTileRangesMax = 1000;
+struct TileRanges {
+  uint64_t begin[kTileRangesMax];
+  uint64_t end[kTileRangesMax];
+  uint64_t first[kTileRangesMax + 1];
+  uint64_t tile_size;
+  int n_ranges;
+};
+cudaError_t launch_tile_expand(const TileRanges &r, uint64_t *tiles, cudaStream_t s);
 // keys: workspace of chunk_sort_size(n_chunks) uint64.
 uint64_t chunk_sort_size(uint64_t n_chunks);
 cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uint32_t *map,

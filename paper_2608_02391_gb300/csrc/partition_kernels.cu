@@ -267,6 +267,34 @@ cudaError_t launch_random_chunk_map(uint64_t n_chunks, int K, uint64_t seed, uin
   return cudaGetLastError();
 }
 
+// Tile table of a list of disjoint ranges, written on the device: tile t lies in the range
+// r with first[r] <= t < first[r + 1] and covers [begin[r] + (t - first[r]) tile_size,
+// min(that + tile_size, end[r])).  The ranges travel in the launch's parameters, so no
+// host staging of the table is needed.
+__global__ void __launch_bounds__(256) tile_expand_kernel(const __grid_constant__ TileRanges a, uint64_t *tiles) {
+  for (uint64_t t = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; t < a.first[a.n_ranges];
+       t += (uint64_t)gridDim.x * blockDim.x) {
+    int lo = 0, hi = a.n_ranges - 1;  // the last range whose first tile is <= t
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.first[mid] <= t) lo = mid;
+      else hi = mid - 1;
+    }
+    const uint64_t b = a.begin[lo] + (t - a.first[lo]) * a.tile_size;
+    const uint64_t e = min(b + a.tile_size, a.end[lo]);
+    reinterpret_cast<ulonglong2 *>(tiles)[t] = make_ulonglong2(b, e);
+  }
+}
+
+cudaError_t launch_tile_expand(const TileRanges &r, uint64_t *tiles, cudaStream_t s) {
+  const uint64_t n = r.first[r.n_ranges];
+  if (n == 0) return cudaSuccess;
+  const uint64_t want = (n + 255) / 256;
+  const unsigned blocks = (unsigned)(want < 4096 ? want : 4096);
+  tile_expand_kernel<<<blocks, 256, 0, s>>>(r, tiles);
+  return cudaGetLastError();
+}
+
 unsigned read_and_clear_partition_errors() {
   unsigned v = 0, zero = 0;
   cudaMemcpyFromSymbol(&v, g_partition_error, sizeof(v));
