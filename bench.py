@@ -478,7 +478,7 @@ def main():
 
     def step(s, events=None):
         for k in range(wl.K):
-            rebuild(k)
+            es._timed(events, "rebuild", lambda: rebuild(k))  # one tile-expansion kernel
             es.round_robin_visit(arena, subs[k], k, s, cfg, d, rewards_dev[s * wl.K + k],
                                  fitness_out=fitness, events=events, partner=partners[k])
 
@@ -582,6 +582,7 @@ def main():
                                     "frac_alu": upd_ops / alu_peak,
                                     "ops_per_normal": alu_ops_per_normal, "normals_per_elem": n_normals_update},
             "shape": {"ms": per["shape"], "launches": counts["shape"]},
+            "tile_rebuild": {"ms": per["rebuild"], "launches": counts["rebuild"]},
             **({"perturb_partner": {"ms": per["partner"], "launches": counts["partner"],
                                     "GB/s": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9,
                                     "frac_hbm": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9 / hbm}}
@@ -783,6 +784,19 @@ def philox_block_share(torch, subs, K: int, lists: bool) -> dict:
         same += int((q[1:] == q[:-1]).sum().item())
         pairs += max(q.numel() - 1, 0)
     return {"value": same / max(pairs, 1), "how": "measured on the index lists"}
+
+
+def chunk_map_launches(copes, n_chunks: int) -> int:
+    """Kernels one copes_random_chunk_map call launches: the keys, a bitonic sort of the
+    workspace's N keys (tiles of 4,096 sorted in shared memory, then for every stage k
+    above the tile one global pass per stride >= 4,096 and one tile pass), and the map."""
+    import ctypes
+    n = copes.load().copes_random_chunk_map_workspace_bytes(ctypes.c_uint64(n_chunks)) // 8
+    tile, launches, k = 4096, 2, 8192
+    while k <= n:
+        launches += (k.bit_length() - 1) - (tile.bit_length() - 1) + 1
+        k <<= 1
+    return launches + 1
 
 
 def host_link_gbs(torch, nbytes=1 << 30, reps=5):
@@ -990,7 +1004,10 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
         },
         "clocks": clk,
         "e2e": None,
-        "gpu_launches": sum(v for k, v in counts.items() if k != "partition"),
+        # each timed partition build launches the random-chunk map's kernels (keys, bitonic
+        # sort, map); its tile tables (over 1,000 ranges each) are copied, not launched
+        "gpu_launches": sum(v for k, v in counts.items() if k != "partition")
+        + counts.get("partition", 0) * chunk_map_launches(copes, -(-layout.d_pad // chunk)),
     }
     print(json.dumps(out), flush=True)
 
