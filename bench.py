@@ -62,7 +62,7 @@ FALLBACK_HBM_GBS = 6800.0
 # The pair perturb's figure comes from subspaces of 2^28 parameters, where the writes still
 # in L2 when the kernel ends are about 2% of its traffic.
 NCU_TRAFFIC = {
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "e98acb47d0b938ec",
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "dc47c2eb721dab12",
                      "bytes_per_elem": 7.827, "capture": "profiles/perturb_pair_4b_slice.md",
                      "case": "two 2^28-parameter subspaces (--case 4b-slice-big)"},
     "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "35ede1dfa8ae5289",
