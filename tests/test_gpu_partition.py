@@ -85,3 +85,21 @@ def test_hash_lists_bit_exact(copes, K):
         assert np.array_equal(got, ref), k
         total += got.size
     assert total == sum(numel)
+
+
+@pytest.mark.parametrize("n_ranges", [1, 999, 1000, 1001, 3000])
+@pytest.mark.parametrize("tile", [1, 777, 4096])
+def test_tile_tables_either_side_of_the_device_expansion_limit(copes, n_ranges, tile):
+    """Up to 1,000 ranges the table is written by a device kernel, beyond that it is split
+    on the host and copied: both give every range cut into [b + i tile, min(b + (i+1)
+    tile, e)) pieces, in range order, bit for bit."""
+    rng = np.random.default_rng(n_ranges * 7 + tile)
+    lens = rng.integers(1, 3 * tile + 5, n_ranges) if tile > 1 else rng.integers(1, 6, n_ranges)
+    gaps = rng.integers(1, 50, n_ranges)  # ranges apart, so none merge
+    b = np.cumsum(gaps + np.concatenate([[0], lens[:-1]])).astype(np.int64) + (1 << 33)
+    ranges = [(int(x), int(x + l)) for x, l in zip(b, lens)]
+    expected = np.array([(s, min(s + tile, e)) for s0, e in ranges for s in range(s0, e, tile)], dtype=np.int64)
+    sub = copes.tiles_from_ranges(ranges, tile_size=tile)
+    torch.cuda.synchronize()
+    got = sub.tensor.cpu().numpy().astype(np.int64).reshape(-1, 2)
+    assert np.array_equal(got, expected)
