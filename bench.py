@@ -3,7 +3,7 @@
 
 Workload: 4B-parameter decoder-shaped set (36 layers, hidden 2560, MLP 9728, vocab 151936,
 tied embeddings; 4,022,468,096 parameters), bf16 working weights + fp32 master (24 GB
-resident, plus an 8 GB second working copy by default), K = 8 layer-block subspaces,
+resident, plus three more 8 GB working copies by default), K = 8 layer-block subspaces,
 N = 32 antithetic members, sigma = 1e-3, alpha = 5e-4, z-score shaping, step coefficient
 alpha / (N sigma).
 
@@ -12,9 +12,10 @@ tile table (the partition step), perturb the 32 members (rewards are seeded synt
 scalars, no model is evaluated), restore, fitness shaping and the fused update + context
 commit.  Every parameter passes through 32 member perturbations, one restore and one
 update per step, so value = parameters per step x steps / time.  `--weights` picks how
-the members are materialised: `dual` (default) writes antithetic members 2j and 2j+1 to
-two working copies in one pass; `partner` keeps one copy and copies member 2j+1 in from
-a partner buffer; `single` perturbs every member from theta.
+the members are materialised: `quad` (default) writes antithetic members 4m .. 4m+3 (two
+noise vectors) to four working copies in one pass; `dual` writes members 2j and 2j+1 to
+two copies in one pass; `partner` keeps one copy and copies member 2j+1 in from a partner
+buffer; `single` perturbs every member from theta.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl copes|reference]
 
@@ -71,6 +72,8 @@ NCU_TRAFFIC = {
 
 
 WEIGHTS_MODES = {
+    "quad": "four bf16 copies: antithetic members 4m, 4m+1 (noise 2m) and 4m+2, 4m+3 (noise 2m+1) evaluated "
+            "on w, w2, w3, w4, all four written by one two-pairs perturb",
     "dual": "two bf16 copies: antithetic member 2j evaluated on w, 2j+1 on w2, both written by one pair perturb",
     "partner": "one bf16 copy: member 2j+1 copied in from the pair perturb's partner buffer",
     "single": "one bf16 copy: every member perturbed from theta",
@@ -87,10 +90,13 @@ def parse():
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
-    ap.add_argument("--weights", default="dual", choices=["dual", "partner", "single"],
-                    help="dual: two working-weight copies, antithetic members 2j on w and 2j+1 on w2 "
-                         "(one pair perturb per pair); partner: one copy, member 2j+1 copied in from a "
-                         "partner buffer; single: one copy, every member perturbed from theta")
+    ap.add_argument("--weights", default=None, choices=["quad", "dual", "partner", "single"],
+                    help="quad (default for tile subspaces): four working-weight copies, two antithetic "
+                         "pairs written by one pass; dual (default for the hash and backup cases): two "
+                         "working-weight copies, antithetic members 2j on w and 2j+1 on w2 (one pair "
+                         "perturb per pair; the backup case keeps one copy and a partner buffer); partner: "
+                         "one copy, member 2j+1 copied in from a partner buffer; single: one copy, every "
+                         "member perturbed from theta")
     ap.add_argument("--cpu-cores", type=int, default=0,
                     help="processes of the oracle's CPU sample (0: every core this process may use)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -407,9 +413,19 @@ def workload_config(wl, args):
 
 
 # -------------------------------------------------------------------------- GPU leg
-def make_arena(copes, torch, wl, layout, dual=False):
+def n_copies(args) -> int:
+    """Working-weight copies of --weights."""
+    return {"quad": 4, "dual": 2}.get(args.weights, 1)
+
+
+def perturb_kernel(args) -> str:
+    """The member perturb --weights times (an N that is a multiple of 4 under quad)."""
+    return {"quad": "perturb_two_pairs", "single": "perturb"}.get(args.weights, "perturb_pair")
+
+
+def make_arena(copes, torch, wl, layout, copies=1):
     """Seeded synthetic weights: fp32 master ~ N(0, init_scale^2), norm tensors 1.0, and
-    w = bf16(master) (and w2 = w for two working copies)."""
+    w = bf16(master) (and the further working copies = w)."""
     master = torch.empty(layout.d_pad, dtype=torch.float32, device="cuda")
     gen = torch.Generator(device="cuda")
     gen.manual_seed(wl.init_seed)
@@ -419,13 +435,15 @@ def make_arena(copes, torch, wl, layout, dual=False):
         if ten.kind == "norm":
             master[int(offs[t]):int(offs[t]) + ten.numel].fill_(1.0)
     w = master.to(torch.bfloat16)
-    return copes.Arena(w, master, w2=w.clone() if dual else None)
+    return copes.Arena(w, master, *[w.clone() for _ in range(copies - 1)])
 
 
 def main():
     args = parse()
     from paper_2608_02391_gb300 import workloads
     wl = workloads.workload({"4b-backup": "4b", "4b-sync": "4b", "4b-backup-slice": "4b-slice"}.get(args.case, args.case))
+    if args.weights is None:
+        args.weights = "dual" if wl.mode == "hash" or args.case in ("4b-backup", "4b-backup-slice") else "quad"
     if args.impl == "reference":
         return run_reference(args, wl)
 
@@ -437,6 +455,8 @@ def main():
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     copes.load()
+    if args.weights == "quad" and (wl.mode == "hash" or args.case in ("4b-backup", "4b-backup-slice")):
+        raise SystemExit("--weights quad needs tile subspaces and an fp32 master: not for --case " + args.case)
     if wl.mode == "hash":
         return run_hash(args, wl, copes, es, torch, rank, world, local)
     if args.case in ("4b-backup", "4b-backup-slice"):
@@ -446,7 +466,7 @@ def main():
 
     layout = copes.Layout(wl.numel)
     d = wl.d
-    arena = make_arena(copes, torch, wl, layout, dual=args.weights == "dual")
+    arena = make_arena(copes, torch, wl, layout, copies=n_copies(args))
     cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping=wl.shaping)
     total_steps = args.warmup + args.steps + args.e2e_steps
     rewards_host = workloads.reward_stream(wl, total_steps * wl.K)  # [steps*K, N]
@@ -457,7 +477,9 @@ def main():
     tile_buf = [s.tensor for s in subs]
     # antithetic pairs: one noise generation per pair, the partner's weights staged in a
     # buffer as wide as the widest subspace
-    if args.weights == "dual":
+    if args.weights == "quad":
+        partners = [es.Partner.four_copies(arena)] * wl.K
+    elif args.weights == "dual":
         partners = [es.Partner.second_copy(arena)] * wl.K
     elif args.weights == "partner":
         partners = es.Partner.per_subspace(arena, subs)
@@ -532,16 +554,17 @@ def main():
     mean_dk = float(np.mean(d_k))
     peaks, peak_src = measured_peaks()
     hbm = float(peaks["hbm_gbs"])
-    paired = args.weights != "single"
-    dual = args.weights == "dual"
+    copies = n_copies(args)
+    pk = perturb_kernel(args)
     # the pair perturb reads theta (4 B) and writes w and the partner's weights (2 + 2 B);
-    # the partner copy reads and writes 2 B; a plain perturb reads 4 B and writes 2 B.
-    # With two working copies, restore and the fused commit write both (+2 B each).
-    perturb_bytes = (8.0 if paired else 6.0) * mean_dk
-    restore_bytes = (8.0 if dual else 6.0) * mean_dk
-    update_bytes = (12.0 if dual else 10.0) * mean_dk
+    # the two-pairs perturb reads theta and writes four copies (4 + 4 x 2 B); the partner
+    # copy reads and writes 2 B; a plain perturb reads 4 B and writes 2 B.  Restore and
+    # the fused commit write every working copy (2 B each).
+    perturb_bytes = {"perturb_two_pairs": 12.0, "perturb_pair": 8.0, "perturb": 6.0}[pk] * mean_dk
+    restore_bytes = (4.0 + 2.0 * copies) * mean_dk
+    update_bytes = (8.0 + 2.0 * copies) * mean_dk
     achieved = perturb_bytes / (per["perturb"] * 1e-3) / 1e9
-    ncu = NCU_TRAFFIC["perturb_pair" if paired else "perturb"]
+    ncu = NCU_TRAFFIC.get(pk, {"source_sha": None})
     traffic = None
     if ncu["source_sha"] == source_sha() and ncu["bytes_per_elem"]:
         traffic = ncu["bytes_per_elem"] * mean_dk
@@ -556,7 +579,9 @@ def main():
     sm_mhz = clk["sm_mhz"] or float(peaks.get("sm_max_mhz", 2070.0))
     alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12  # Tops/s at the sampled clock
     upd_ops = mean_dk * n_normals_update * alu_ops_per_normal / (per["update"] * 1e-3) / 1e12
-    bytes_per_step = d * ((wl.n_members // 2) * 8 + 8 + 12 if dual else wl.n_members * 6 + 6 + 10)
+    members_bytes = {"perturb_two_pairs": (wl.n_members // 4) * 12, "perturb_pair": (wl.n_members // 2) * 8,
+                     "perturb": wl.n_members * 6}[pk] + (wl.n_members // 2) * 4 * (args.weights == "partner")
+    bytes_per_step = d * (members_bytes + (4 + 2 * copies) + (8 + 2 * copies))
     value = job_throughput(world, d, args.steps, ms * 1e-3)
     e2e = job_throughput(world, d, args.e2e_steps, e2e_s)
     launches = sum(counts.values())
@@ -566,13 +591,15 @@ def main():
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": workload_config(wl, args),
         "hbm_gbs": bytes_per_step * args.steps / (ms * 1e-3) / 1e9,
-        "roofline": {"bound": "hbm", "kernel": "perturb_pair" if paired else "perturb", "achieved": achieved,
+        "roofline": {"bound": "hbm", "kernel": pk, "achieved": achieved,
                      "peak": hbm, "unit": "GB/s", "frac": achieved / hbm, "traffic": traffic,
                      "traffic_source": traffic_note,
                      "peak_source": peak_src, "algorithmic_bytes_per_launch": perturb_bytes},
         "kernels": {
-            ("perturb_pair" if paired else "perturb"): {
-                "ms": per["perturb"], "launches": counts["perturb"], "GB/s": achieved, "frac_hbm": achieved / hbm},
+            pk: {"ms": per["perturb"], "launches": counts["perturb"], "GB/s": achieved, "frac_hbm": achieved / hbm,
+                 # pinned lane-ops: 27 per normal, 3 per member written (fma, round, pack)
+                 **({"frac_alu": (2 * 27 + 4 * 3) * mean_dk / (per["perturb"] * 1e-3) / (alu_peak * 1e12),
+                     "ops_per_elem": 2 * 27 + 4 * 3} if pk == "perturb_two_pairs" else {})},
             "restore": {"ms": per["restore"], "launches": counts["restore"],
                         "GB/s": restore_bytes / (per["restore"] * 1e-3) / 1e9,
                         "frac_hbm": restore_bytes / (per["restore"] * 1e-3) / 1e9 / hbm},
@@ -625,7 +652,7 @@ def run_hash(args, wl, copes, es, torch, rank, world, local):
     from paper_2608_02391_gb300 import workloads
     layout = copes.Layout(wl.numel, list(range(len(wl.tensors))))
     d = wl.d
-    arena = make_arena(copes, torch, wl, layout, dual=args.weights == "dual")
+    arena = make_arena(copes, torch, wl, layout, copies=n_copies(args))
     # a hash subspace spreads over the whole arena: the partner is w2 or a full-size buffer
     if args.weights == "dual":
         partner = es.Partner.second_copy(arena)
@@ -914,7 +941,7 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
     K, chunk = 4, 65536
     layout = copes.Layout(wl.numel)
     d = wl.d
-    arena = make_arena(copes, torch, wl, layout, dual=args.weights == "dual")
+    arena = make_arena(copes, torch, wl, layout, copies=n_copies(args))
     cfg = es.ESConfig(n_members=wl.n_members, sigma=wl.sigma, alpha=wl.alpha, shaping="zscore",
                       convention=copes.COEF_PAPER, dimension_aware=True)
     total = args.warmup + args.steps
@@ -923,7 +950,9 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
     # each step's partition is built on a side stream while the previous step runs
     parts = es.ChunkPrefetcher(layout, K, lambda s: 1000 + s, chunk=chunk, tile_size=args.tile)
     # random chunks spread every subspace over the arena: one partner buffer covers it
-    if args.weights == "dual":
+    if args.weights == "quad":
+        partner = es.Partner.four_copies(arena)
+    elif args.weights == "dual":
         partner = es.Partner.second_copy(arena)
     elif args.weights == "partner":
         partner = es.Partner(torch.empty(layout.d_pad, dtype=arena.w.dtype, device="cuda"), 0)
@@ -965,12 +994,13 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
     alu_peak = props.multi_processor_count * 128 * sm_mhz * 1e6 / 1e12
     P = (wl.n_members // K) // 2
     upd_tops = 28.0 * P * mean_dk / (per["update"] * 1e-3) / 1e12
-    upd_gbs = 10.0 * mean_dk / (per["update"] * 1e-3) / 1e9
+    upd_bytes = 8.0 + 2.0 * n_copies(args)  # read and write theta, write every working copy
+    upd_gbs = upd_bytes * mean_dk / (per["update"] * 1e-3) / 1e9
     # the update's roofline is the slower of its ALU and HBM bounds
     t_alu = 28.0 * P * mean_dk / (alu_peak * 1e12)
-    t_hbm = 10.0 * mean_dk / (hbm * 1e9)
-    paired = args.weights != "single"
-    perturb_gbs = (8.0 if paired else 6.0) * mean_dk / (per["perturb"] * 1e-3) / 1e9
+    t_hbm = upd_bytes * mean_dk / (hbm * 1e9)
+    pk = perturb_kernel(args)
+    perturb_gbs = {"perturb_two_pairs": 12.0, "perturb_pair": 8.0, "perturb": 6.0}[pk] * mean_dk / (per["perturb"] * 1e-3) / 1e9
     value = job_throughput(world, d, args.steps, ms * 1e-3)
     out = {
         "metric": METRIC, "value": value, "unit": "params/s", "n_gpus": world, "steps": args.steps,
@@ -982,20 +1012,20 @@ def run_sync(args, wl, copes, es, torch, rank, world, local):
                    "params": d, "K": K, "N": wl.n_members, "chunk": chunk, "sigma": wl.sigma, "alpha": wl.alpha,
                    "tile": args.tile, "working_weights": WEIGHTS_MODES[args.weights],
                    "l2": "inputs larger than L2, no flush"},
-        "roofline": {"bound": "hbm", "kernel": "perturb_pair" if paired else "perturb", "achieved": perturb_gbs,
+        "roofline": {"bound": "hbm", "kernel": pk, "achieved": perturb_gbs,
                      "peak": hbm, "unit": "GB/s", "frac": perturb_gbs / hbm, "traffic": None,
                      "peak_source": "measured"},
         "kernels": {
             "partition": {"ms": per.get("partition"), "launches": counts.get("partition", 0),
                           "note": "side-stream window, host tile building included; overlapped with "
                                   "the previous step"},
-            ("perturb_pair" if paired else "perturb"): {"ms": per["perturb"], "launches": counts["perturb"],
-                                                        "GB/s": perturb_gbs, "frac_hbm": perturb_gbs / hbm},
+            pk: {"ms": per["perturb"], "launches": counts["perturb"], "GB/s": perturb_gbs,
+                 "frac_hbm": perturb_gbs / hbm},
             **({"perturb_partner": {"ms": per["partner"], "launches": counts["partner"],
                                     "GB/s": 4.0 * mean_dk / (per["partner"] * 1e-3) / 1e9}}
                if "partner" in per else {}),
             "restore": {"ms": per["restore"], "launches": counts["restore"],
-                        "GB/s": 6.0 * mean_dk / (per["restore"] * 1e-3) / 1e9},
+                        "GB/s": (4.0 + 2.0 * n_copies(args)) * mean_dk / (per["restore"] * 1e-3) / 1e9},
             "update_fused_commit": {"ms": per["update"], "launches": counts["update"], "Tops": upd_tops,
                                     "GB/s": upd_gbs, "normals_per_elem": P,
                                     "frac_of_slower_bound": max(t_alu, t_hbm) / (per["update"] * 1e-3),

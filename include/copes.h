@@ -79,19 +79,26 @@ enum {
  * w2 (optional, NULL for none) is a second working-weight buffer of the same dtype and
  * size, for evaluating the two members of an antithetic pair on two copies of the model:
  * copes_perturb_pair with partner = w2, partner_base = 0, partner_len = n_alloc writes
- * member 2j's weights to w and member 2j+1's to w2 in one pass.  Restore, commit, the
- * fused update's commit and init then write the context to w2 as well as w, so outside
- * the live subspace both buffers always hold the context.  Perturbs write w only. */
+ * member 2j's weights to w and member 2j+1's to w2 in one pass.  w3 and w4 (optional,
+ * set together and only with w2) make four copies, on which copes_perturb_two_pairs
+ * writes the four members of two antithetic pairs in one pass.  Restore, commit, the
+ * fused update's commit and init write the context to every copy, so outside the live
+ * subspace all of them always hold the context.  Perturbs write only the copies their
+ * call names. */
 typedef struct {
   void *w;          /* device: working weights, n_alloc elements of dtype              */
   float *master;    /* device: fp32 master theta, n_alloc elements                     */
   uint64_t n_alloc; /* elements in each buffer; every subspace index must be < n_alloc */
   int dtype;        /* COPES_BF16 or COPES_FP32 (the dtype of w)                       */
   void *w2;         /* device, optional: second working buffer (16-byte aligned), or NULL */
+  void *w3;         /* device, optional: third working buffer (16-byte aligned), or NULL  */
+  void *w4;         /* device, optional: fourth working buffer (16-byte aligned), or NULL */
 } copes_params;
-/* w, master and w2 must be pairwise disjoint byte ranges (n_alloc elements each): the
- * kernels read the master while they write the working buffers.  Every call that takes
- * copes_params checks this and returns COPES_ERR_INVALID_ARG otherwise. */
+/* w, master, w2, w3 and w4 must be pairwise disjoint byte ranges (n_alloc elements
+ * each): the kernels read the master while they write the working buffers.  Every call
+ * that takes copes_params checks this, and that w3 and w4 come together and only with
+ * w2, and returns COPES_ERR_INVALID_ARG otherwise.  A caller that zero-initialises the
+ * struct and sets the first five fields gets one or two copies, as before w3 and w4. */
 
 /* A subspace S (Eq. 7 / Eq. 8: the support of P_k).
  *  TILES:       a device array of n_tiles [begin, end) pairs of uint64 global indices
@@ -340,14 +347,27 @@ int copes_perturb_pair(const copes_params *p, const copes_subspace *S, uint64_t 
 int copes_perturb_partner(const copes_params *p, const copes_subspace *S, const void *partner,
                           uint64_t partner_base, uint64_t partner_len, cudaStream_t stream);
 
+/* Two antithetic pairs in one pass (Eq. 8 for the four members of two noise vectors; no
+ * counterpart in the paper's implementation).  With four working copies (p->w2, p->w3
+ * and p->w4 set), for every g in S:
+ *   w[g]  = round(fma( signed_sigma, eps_seed_a[g], theta[g]))
+ *   w2[g] = round(fma(-signed_sigma, eps_seed_a[g], theta[g]))
+ *   w3[g] = round(fma( signed_sigma, eps_seed_b[g], theta[g]))
+ *   w4[g] = round(fma(-signed_sigma, eps_seed_b[g], theta[g]))
+ * each exactly what copes_perturb writes with that seed and signed sigma, from one read
+ * of theta.  Elements outside S are untouched.  TILES subspaces only
+ * (COPES_ERR_UNSUPPORTED otherwise); without four copies COPES_ERR_INVALID_ARG. */
+int copes_perturb_two_pairs(const copes_params *p, const copes_subspace *S, uint64_t seed_a,
+                            uint64_t seed_b, float signed_sigma, cudaStream_t stream);
+
 /* Restore (Sec. 3.3, Supp. A.8 "CPU Weight Backup", here an on-device fp32 master):
- *   w[g] = round(theta[g]) for g in S, bit-exact; outside S untouched.  With p->w2 set,
- * w2[g] gets the same value. */
+ *   w[g] = round(theta[g]) for g in S, bit-exact; outside S untouched.  Every further
+ * working copy (w2, w3, w4) that p sets gets the same value. */
 int copes_restore(const copes_params *p, const copes_subspace *S, cudaStream_t stream);
 
 /* Context commit (Sec. 3.2 shared context after Eq. 13): w[g] = round(theta[g]) for
- * g in S (and w2[g] with p->w2 set).  Same arithmetic as copes_restore, called after
- * copes_update. */
+ * g in S (and in every further working copy p sets).  Same arithmetic as copes_restore,
+ * called after copes_update. */
 int copes_context_commit(const copes_params *p, const copes_subspace *S, cudaStream_t stream);
 
 /* Fitness shaping (Eq. 5, Eq. 12, Sec. 4.4): f = shape(r) over n rewards (device fp32),
@@ -362,15 +382,16 @@ int copes_shape_fitness(const float *rewards, int n, const int32_t *group, int m
  * All n_noise noise vectors are regenerated in registers in one pass; nothing is
  * stored.  noise_id, sign (host, n_members) and seeds (host, n_noise) are read during
  * the call; fitness is device fp32 [n_members].  fuse_commit != 0 also writes
- * w[g] = round(theta[g]) (the context commit; w2[g] too with p->w2 set) in the same
- * pass. */
+ * w[g] = round(theta[g]) (the context commit, to every working copy p sets) in the
+ * same pass. */
 int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
                  const int32_t *noise_id, const int8_t *sign, const float *fitness,
                  int n_noise, const uint64_t *seeds, float coef, int fuse_commit,
                  cudaStream_t stream);
 
 /* Synthetic initialisation (input preparation, not part of the method): for g in S,
- *   theta[g] = mean + scale * eps_seed^(INIT)[g],  w[g] = round(theta[g])  (and w2[g]). */
+ *   theta[g] = mean + scale * eps_seed^(INIT)[g],  w[g] = round(theta[g])  (and every
+ * further working copy). */
 int copes_init_normal(const copes_params *p, const copes_subspace *S, uint64_t seed,
                       float mean, float scale, cudaStream_t stream);
 

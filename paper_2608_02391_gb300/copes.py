@@ -42,7 +42,8 @@ class CopesError(RuntimeError):
 
 class Params(ctypes.Structure):
     _fields_ = [("w", ctypes.c_void_p), ("master", ctypes.c_void_p), ("n_alloc", ctypes.c_uint64),
-                ("dtype", ctypes.c_int), ("w2", ctypes.c_void_p)]
+                ("dtype", ctypes.c_int), ("w2", ctypes.c_void_p), ("w3", ctypes.c_void_p),
+                ("w4", ctypes.c_void_p)]
 
 
 class Subspace(ctypes.Structure):
@@ -94,6 +95,7 @@ SIGNATURES = {
     "copes_perturb": (_I32, [_VP, _VP, _U64, _F32, _VP]),
     "copes_perturb_pair": (_I32, [_VP, _VP, _U64, _F32, _VP, _U64, _U64, _VP]),
     "copes_perturb_partner": (_I32, [_VP, _VP, _VP, _U64, _U64, _VP]),
+    "copes_perturb_two_pairs": (_I32, [_VP, _VP, _U64, _U64, _F32, _VP]),
     "copes_restore": (_I32, [_VP, _VP, _VP]),
     "copes_context_commit": (_I32, [_VP, _VP, _VP]),
     "copes_shape_fitness": (_I32, [_VP, _I32, _VP, _I32, _VP, _VP]),
@@ -207,21 +209,30 @@ class Layout:
 # ----------------------------------------------------------------------------- arena
 class Arena:
     """The flat parameter arena: working weights w (bf16 or fp32) and the fp32 master, and
-    optionally a second working buffer w2 (copes_params.w2) that restore, commit and init
-    keep equal to w outside the live member's perturbation.  `live` is the working buffer
-    that holds the member being evaluated (w, or w2 for a pair's second member when w2
-    serves as the partner buffer)."""
+    optionally further working copies -- w2 (copes_params.w2), or w2, w3 and w4 -- that
+    restore, commit and init keep equal to w outside the live members' perturbations.
+    `live` is the working buffer that holds the member being evaluated (w, or the copy a
+    pair's or two pairs' perturb wrote that member to)."""
 
-    def __init__(self, w: torch.Tensor, master: torch.Tensor, w2: Optional[torch.Tensor] = None):
+    def __init__(self, w: torch.Tensor, master: torch.Tensor, w2: Optional[torch.Tensor] = None,
+                 w3: Optional[torch.Tensor] = None, w4: Optional[torch.Tensor] = None):
         assert w.is_cuda and master.is_cuda and w.is_contiguous() and master.is_contiguous()
         assert master.dtype == torch.float32 and w.numel() == master.numel()
-        if w2 is not None:
-            assert w2.is_cuda and w2.is_contiguous() and w2.dtype == w.dtype and w2.numel() == w.numel()
-        self.w, self.master, self.w2 = w, master, w2
+        assert (w3 is None) == (w4 is None) and (w3 is None or w2 is not None), \
+            "w3 and w4 come together, and only with w2"
+        for c in (w2, w3, w4):
+            if c is not None:
+                assert c.is_cuda and c.is_contiguous() and c.dtype == w.dtype and c.numel() == w.numel()
+        self.w, self.master, self.w2, self.w3, self.w4 = w, master, w2, w3, w4
         self.live = w
         dt = {torch.bfloat16: BF16, torch.float32: FP32}[w.dtype]
-        self.params = Params(w.data_ptr(), master.data_ptr(), w.numel(), dt,
-                             None if w2 is None else w2.data_ptr())
+        ptr = lambda c: None if c is None else c.data_ptr()
+        self.params = Params(w.data_ptr(), master.data_ptr(), w.numel(), dt, ptr(w2), ptr(w3), ptr(w4))
+
+    @property
+    def copies(self) -> List[torch.Tensor]:
+        """The working copies in order: [w], [w, w2] or [w, w2, w3, w4]."""
+        return [c for c in (self.w, self.w2, self.w3, self.w4) if c is not None]
 
     @classmethod
     def empty(cls, n: int, dtype=torch.bfloat16, device="cuda"):
@@ -410,6 +421,16 @@ def perturb_pair(arena: Arena, sub: SubspaceHandle, seed: int, signed_sigma: flo
     S = sub.struct()
     _check(load().copes_perturb_pair(ctypes.byref(arena.params), ctypes.byref(S), seed, signed_sigma,
                                      _ptr(partner), base, view.numel(), _stream(stream)))
+
+
+def perturb_two_pairs(arena: Arena, sub: SubspaceHandle, seed_a: int, seed_b: int, signed_sigma: float,
+                      stream=None) -> None:
+    """copes_perturb_two_pairs: w = perturb(seed_a, +s), w2 = perturb(seed_a, -s),
+    w3 = perturb(seed_b, +s), w4 = perturb(seed_b, -s) in one pass (four working copies,
+    TILES subspaces)."""
+    S = sub.struct()
+    _check(load().copes_perturb_two_pairs(ctypes.byref(arena.params), ctypes.byref(S), seed_a, seed_b,
+                                          signed_sigma, _stream(stream)))
 
 
 def perturb_partner(arena: Arena, sub: SubspaceHandle, partner: torch.Tensor, base: int = 0,

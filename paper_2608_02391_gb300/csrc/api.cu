@@ -54,17 +54,40 @@ int check_params(const copes_params *p, const char *who) {
                 p->dtype);
   if (!aligned(p->w, 16) || !aligned(p->master, 16))
     return fail(COPES_ERR_ALIGNMENT, "%s: w and master must be 16-byte aligned", who);
-  if (p->w2 && !aligned(p->w2, 16)) return fail(COPES_ERR_ALIGNMENT, "%s: w2 must be 16-byte aligned", who);
-  if (p->w2 && (p->w2 == p->w || p->w2 == (void *)p->master))
-    return fail(COPES_ERR_INVALID_ARG, "%s: w2 must be a buffer of its own", who);
+  if ((p->w3 == nullptr) != (p->w4 == nullptr))
+    return fail(COPES_ERR_INVALID_ARG, "%s: w3 and w4 are set together", who);
+  if (p->w3 && !p->w2) return fail(COPES_ERR_INVALID_ARG, "%s: w3 and w4 need w2", who);
+  if (!aligned(p->w2, 16) || !aligned(p->w3, 16) || !aligned(p->w4, 16))
+    return fail(COPES_ERR_ALIGNMENT, "%s: w2, w3 and w4 must be 16-byte aligned", who);
   if (p->n_alloc == 0) return fail(COPES_ERR_SIZE, "%s: n_alloc is 0", who);
-  // the kernels read master while they write w (and w2): the three must be disjoint
+  // the kernels read master while they write the working copies: all must be disjoint
   const uint64_t wbytes = p->n_alloc * elem_size(p->dtype), mbytes = p->n_alloc * 4;
   if (overlaps(p->w, wbytes, p->master, mbytes))
     return fail(COPES_ERR_INVALID_ARG, "%s: w and master overlap", who);
-  if (p->w2 && (overlaps(p->w2, wbytes, p->w, wbytes) || overlaps(p->w2, wbytes, p->master, mbytes)))
-    return fail(COPES_ERR_INVALID_ARG, "%s: w2 overlaps w or master", who);
+  const void *extra[3] = {p->w2, p->w3, p->w4};
+  static const char *name[3] = {"w2", "w3", "w4"};
+  for (int i = 0; i < 3; ++i) {
+    if (!extra[i]) continue;
+    if (extra[i] == p->w || extra[i] == (const void *)p->master)
+      return fail(COPES_ERR_INVALID_ARG, "%s: %s must be a buffer of its own", who, name[i]);
+    if (overlaps(extra[i], wbytes, p->w, wbytes) || overlaps(extra[i], wbytes, p->master, mbytes))
+      return fail(COPES_ERR_INVALID_ARG, "%s: %s overlaps w or master", who, name[i]);
+    for (int j = 0; j < i; ++j)
+      if (extra[j] && (extra[j] == extra[i] || overlaps(extra[i], wbytes, extra[j], wbytes)))
+        return fail(COPES_ERR_INVALID_ARG, "%s: %s overlaps %s", who, name[i], name[j]);
+  }
   return COPES_OK;
+}
+
+// The working copies beyond w, in order: none, w2, or w2, w3, w4 (check_params enforces
+// that w3 and w4 come together and only with w2).
+copes::WorkingCopies working_copies(const copes_params *p) {
+  copes::WorkingCopies c{};
+  c.p[0] = p->w2;
+  c.p[1] = p->w3;
+  c.p[2] = p->w4;
+  c.n = p->w4 ? 3 : (p->w2 ? 1 : 0);
+  return c;
 }
 
 int check_subspace(const copes_subspace *S, const char *who) {
@@ -155,7 +178,7 @@ int launch_status(cudaError_t e, const char *who) {
 ElemArgs elem_args(const copes_params *p, const copes_subspace *S) {
   ElemArgs a{};
   a.w = p->w;
-  a.w2 = p->w2;
+  a.copies = working_copies(p);
   a.master = p->master;
   a.n_alloc = p->n_alloc;
   if (S->kind == COPES_SUBSPACE_TILES) {
@@ -190,7 +213,7 @@ struct Partner {
 
 int run_elementwise(int op, const copes_params *p, const copes_subspace *S, uint64_t seed,
                     uint32_t tag, float a_val, float b_val, cudaStream_t s, const char *who,
-                    const Partner &partner = Partner{}) {
+                    const Partner &partner = Partner{}, uint64_t seed_b = 0) {
   int rc = check_params(p, who);
   if (rc) return rc;
   if ((rc = check_subspace(S, who))) return rc;
@@ -206,6 +229,11 @@ int run_elementwise(int op, const copes_params *p, const copes_subspace *S, uint
   // the scale folded into the normal's polynomial: a * eps = x * (a * R(L))
   scaled_coeffs(a_val, a.coeffs);
   copes::philox_round_keys(a.seed_lo, a.seed_hi, a.rk);
+  if (op == copes::kOpPerturbTwoPairs) {
+    copes::philox_round_keys((uint32_t)seed_b, (uint32_t)(seed_b >> 32), a.rk_b);
+    copes::philox_folded_keys(a.rk, tag, a.fk);
+    copes::philox_folded_keys(a.rk_b, tag, a.fk_b);
+  }
   if (S->kind == COPES_SUBSPACE_HASH_REPLAY)
     return launch_status(copes::launch_replay_elementwise(op, p->dtype, a, replay_args(S), s), who);
   return launch_status(copes::launch_elementwise(op, S->kind, p->dtype, a, s), who);
@@ -614,6 +642,19 @@ int copes_perturb_partner(const copes_params *p, const copes_subspace *S, const 
                          Partner{partner, partner_base, partner_len});
 }
 
+int copes_perturb_two_pairs(const copes_params *p, const copes_subspace *S, uint64_t seed_a,
+                            uint64_t seed_b, float signed_sigma, cudaStream_t stream) {
+  const char *who = "copes_perturb_two_pairs";
+  if (!isfinite(signed_sigma)) return fail(COPES_ERR_INVALID_ARG, "%s: sigma is not finite", who);
+  int rc = check_params(p, who);
+  if (rc) return rc;
+  if (!p->w4) return fail(COPES_ERR_INVALID_ARG, "%s: needs four working copies (w2, w3 and w4 set)", who);
+  if ((rc = check_subspace(S, who))) return rc;
+  if (S->kind != COPES_SUBSPACE_TILES) return fail(COPES_ERR_UNSUPPORTED, "%s: TILES subspaces only", who);
+  return run_elementwise(copes::kOpPerturbTwoPairs, p, S, seed_a, COPES_TAG_NOISE, signed_sigma, 0.0f, stream,
+                         who, Partner{}, seed_b);
+}
+
 int copes_restore(const copes_params *p, const copes_subspace *S, cudaStream_t stream) {
   return run_elementwise(copes::kOpRestore, p, S, 0, 0, 0.0f, 0.0f, stream, "copes_restore");
 }
@@ -760,7 +801,7 @@ int copes_update(const copes_params *p, const copes_subspace *S, int n_members,
   UpdateArgs a{};
   if ((rc = fill_update_members(a, n_members, noise_id, sign, fitness, n_noise, seeds, coef, who))) return rc;
   a.w = p->w;
-  a.w2 = p->w2;
+  a.copies = working_copies(p);
   a.master = p->master;
   a.n_alloc = p->n_alloc;
   if (S->kind == COPES_SUBSPACE_TILES) {

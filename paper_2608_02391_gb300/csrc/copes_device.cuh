@@ -220,6 +220,50 @@ __device__ __forceinline__ void normal_parts_groups_x2(const uint32_t (&w)[G][4]
   }
 }
 
+// normal_parts_groups_x2 with every step on packed pairs, as in normal_parts_groups_packed
+// but with the caller's scaled coefficients (central2: (c, c) pairs): x2[i][p] and r2[i][p]
+// hold words 2p and 2p + 1 of block i, each value normal_parts_groups_x2's bit for bit.
+template <int G, int NC, int NT>
+__device__ __forceinline__ void normal_parts_groups_x2_packed(const uint32_t (&w)[G][4],
+                                                              const unsigned long long (&central2)[NC],
+                                                              const float (&tail)[NT],
+                                                              unsigned long long (&x2)[G][2],
+                                                              unsigned long long (&r2)[G][2]) {
+  float L[G][4];
+  float L_min = 0.0f;  // L <= 0 for every word
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+#pragma unroll
+    for (int p = 0; p < 2; ++p) {
+      const unsigned long long F = pack_f32x2(__uint_as_float((w[i][2 * p] & 0x007FFFFEu) | 0x40000001u),
+                                              __uint_as_float((w[i][2 * p + 1] & 0x007FFFFEu) | 0x40000001u));
+      x2[i][p] = add_f32x2(F, splat_f32x2(-3.0f));
+      float t0, t1;  // x^2 - 1 = -(1 - x^2)
+      unpack_f32x2(fma_f32x2(x2[i][p], x2[i][p], splat_f32x2(-1.0f)), t0, t1);
+      L[i][2 * p] = lg2_approx(-t0);
+      L[i][2 * p + 1] = lg2_approx(-t1);
+      L_min = fminf(L_min, fminf(L[i][2 * p], L[i][2 * p + 1]));
+      const unsigned long long Lp = pack_f32x2(L[i][2 * p], L[i][2 * p + 1]);
+      unsigned long long acc = central2[NC - 1];
+#pragma unroll
+      for (int k = NC - 2; k >= 0; --k) acc = fma_f32x2(acc, Lp, central2[k]);
+      r2[i][p] = acc;
+    }
+  }
+  if (__any_sync(__activemask(), L_min < COPES_NORMAL_L_SPLIT)) {
+#pragma unroll
+    for (int i = 0; i < G; ++i)
+#pragma unroll
+      for (int p = 0; p < 2; ++p) {
+        float r0, r1;
+        unpack_f32x2(r2[i][p], r0, r1);
+        if (L[i][2 * p] < COPES_NORMAL_L_SPLIT) r0 = tail_ratio(tail, L[i][2 * p]);
+        if (L[i][2 * p + 1] < COPES_NORMAL_L_SPLIT) r1 = tail_ratio(tail, L[i][2 * p + 1]);
+        r2[i][p] = pack_f32x2(r0, r1);
+      }
+  }
+}
+
 // Two standard normals from two words (of different Philox blocks), their central
 // polynomials evaluated as one packed pair with compile-time coefficients and a single
 // warp vote for the tail: bit-identical to two normal_from_word calls.

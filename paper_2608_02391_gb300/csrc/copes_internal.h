@@ -147,6 +147,12 @@ struct ScaledCoeffs {
   float tail[COPES_NORMAL_TAIL_DEGREE + 1];
 };
 
+// The working copies beyond w (copes_params.w2, w3, w4): n = 0, 1 (w2) or 3 (w2, w3, w4).
+struct WorkingCopies {
+  void *p[3];
+  int n;
+};
+
 struct ElemArgs {
   void *w;
   float *master;
@@ -166,12 +172,19 @@ struct ElemArgs {
   // g at partner[g - partner_base] for partner_base <= g < partner_base + partner_len
   void *partner;
   uint64_t partner_base, partner_len;
-  void *w2;  // second working buffer (copes_params.w2) or NULL: restore / commit / init write both
+  WorkingCopies copies;  // restore / commit / init write these as well as w
+  // kOpPerturbTwoPairs: the second noise vector's round keys, and both vectors' folded keys
+  // (philox_folded_keys, noise tag) for counters below 2^32
+  uint32_t rk_b[20];
+  uint32_t fk[20], fk_b[20];
 };
 
 // kOpGather / kOpScatter copy theta between master and the gathered copy (INDICES only).
 // kOpPerturbPair writes w = rn(theta + a eps) and the partner member's rn(theta - a eps)
-// to the partner buffer; kOpPartner copies the partner buffer into w.
+// to the partner buffer; kOpPartner copies the partner buffer into w.  kOpPerturbTwoPairs
+// (TILES only, three further working copies) writes rn(theta + a eps) and
+// rn(theta - a eps) for the first noise vector to w and copies[0], and for the second
+// (keys rk_b) to copies[1] and copies[2].
 enum ElemOp {
   kOpPerturb = 0,
   kOpRestore = 1,
@@ -179,7 +192,8 @@ enum ElemOp {
   kOpGather = 3,
   kOpScatter = 4,
   kOpPerturbPair = 5,
-  kOpPartner = 6
+  kOpPartner = 6,
+  kOpPerturbTwoPairs = 7
 };
 
 struct UpdateArgs {
@@ -201,7 +215,7 @@ struct UpdateArgs {
   uint16_t noise_member[COPES_MAX_MEMBERS];
   int8_t sign[COPES_MAX_MEMBERS];
   float *gathered;  // INDICES: theta in list order instead of master[index[p]] (or NULL)
-  void *w2;         // second working buffer or NULL: the fused commit writes both
+  WorkingCopies copies;  // the fused commit writes these as well as w
 };
 
 // ------------------------------------------------------------------------ launchers

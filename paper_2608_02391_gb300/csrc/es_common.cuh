@@ -36,6 +36,22 @@ struct WStore<float> {
   }
 };
 
+// The context's stores to the working copies beyond w (restore / commit / init and the
+// update's fused commit).
+template <typename WT>
+__device__ __forceinline__ void store_copies_full(const WorkingCopies &c, uint64_t g, const float v[4]) {
+#pragma unroll
+  for (int i = 0; i < 3; ++i)
+    if (i < c.n) WStore<WT>::full(c.p[i], g, v);
+}
+
+template <typename WT>
+__device__ __forceinline__ void store_copies_one(const WorkingCopies &c, uint64_t g, float v) {
+#pragma unroll
+  for (int i = 0; i < 3; ++i)
+    if (i < c.n) WStore<WT>::one(c.p[i], g, v);
+}
+
 // The update's prologue: folds the members into one weight per noise vector,
 //   w_j = sum_{i : noise(i) = j} sign_i f_i  (member order, fp32),
 // and expands each noise vector's Philox round keys into shared memory (and, when s_fk is

@@ -89,6 +89,119 @@ __device__ __forceinline__ void pair_perturb_step(const ElemArgs &a, uint64_t b,
   }
 }
 
+// Two antithetic pairs of the group at counter (q_lo, q_hi) (kOpPerturbTwoPairs):
+// v[0] = theta + a eps_A, v[1] = theta - a eps_A, v[2] = theta + a eps_B and
+// v[3] = theta - a eps_B, each bit for bit what kOpPerturb computes with that noise vector
+// and sign (normal_parts_groups_x2 gives normal_parts4_x2's values).
+__device__ __forceinline__ void two_pairs_values(const ElemArgs &a, uint32_t q_lo, uint32_t q_hi,
+                                                 const float th[4], float (&v)[4][4]) {
+  uint32_t w[2][4];
+  philox4x32_10_rk(q_lo, q_hi, 0u, COPES_TAG_NOISE, a.rk, w[0]);
+  philox4x32_10_rk(q_lo, q_hi, 0u, COPES_TAG_NOISE, a.rk_b, w[1]);
+  float x[2][4], r[2][4];  // r = a * R(L)
+  normal_parts_groups_x2<2>(w, a.coeffs.central2, a.coeffs.tail, x, r);
+#pragma unroll
+  for (int s = 0; s < 2; ++s)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      v[2 * s][e] = __fmaf_rn(r[s][e], x[s][e], th[e]);
+      v[2 * s + 1][e] = __fmaf_rn(-r[s][e], x[s][e], th[e]);
+    }
+}
+
+// The four members' values go to w, copies[0], copies[1] and copies[2].
+template <typename WT>
+__device__ __forceinline__ void store_two_pairs_full(const ElemArgs &a, uint64_t g, const float (&v)[4][4]) {
+  WStore<WT>::full(a.w, g, v[0]);
+  WStore<WT>::full(a.copies.p[0], g, v[1]);
+  WStore<WT>::full(a.copies.p[1], g, v[2]);
+  WStore<WT>::full(a.copies.p[2], g, v[3]);
+}
+
+template <typename WT>
+__device__ __forceinline__ void store_two_pairs_one(const ElemArgs &a, uint64_t g, const float (&v)[4][4], int k) {
+  WStore<WT>::one(a.w, g, v[0][k]);
+  WStore<WT>::one(a.copies.p[0], g, v[1][k]);
+  WStore<WT>::one(a.copies.p[1], g, v[2][k]);
+  WStore<WT>::one(a.copies.p[2], g, v[3][k]);
+}
+
+// One step of the two-pairs perturb over the thread's G groups of an aligned tile whose
+// counters are all below 2^32: each group's product M0 q is computed once and shared by
+// both noise vectors' folded Philox (philox4x32_10_folded, the same words as
+// philox4x32_10_rk), the 2G blocks' transforms take one tail vote, and each group's four
+// members are formed on packed pairs and stored -- two_pairs_values' results, bit for bit
+// (the antithetic member as fma(r, -x, theta): -x is exact).  Groups past the tile's end are
+// generated but not stored.
+template <typename WT, int G>
+__device__ __forceinline__ void two_pairs_step(const ElemArgs &a, uint64_t b, uint32_t len, uint32_t off,
+                                               uint32_t q0_lo, const float (&th)[G][4]) {
+  uint32_t w[2 * G][4];
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+    const uint64_t m = (uint64_t)kPhiloxM0 * (q0_lo + ((off + 4u * kThreads * i) >> 2));
+    philox4x32_10_folded((uint32_t)m, (uint32_t)(m >> 32), a.fk, w[i]);
+    philox4x32_10_folded((uint32_t)m, (uint32_t)(m >> 32), a.fk_b, w[G + i]);
+  }
+  unsigned long long x2[2 * G][2], r2[2 * G][2];
+  normal_parts_groups_x2_packed<2 * G>(w, a.coeffs.central2, a.coeffs.tail, x2, r2);
+#pragma unroll
+  for (int i = 0; i < G; ++i) {
+    const uint32_t o = off + 4u * kThreads * i;
+    if (o >= len) continue;
+    float v[4][4];
+#pragma unroll
+    for (int s = 0; s < 2; ++s)
+#pragma unroll
+      for (int p = 0; p < 2; ++p) {
+        const unsigned long long t2 = pack_f32x2(th[i][2 * p], th[i][2 * p + 1]);
+        const unsigned long long xs = x2[s * G + i][p], rs = r2[s * G + i][p];
+        unpack_f32x2(fma_f32x2(rs, xs, t2), v[2 * s][2 * p], v[2 * s][2 * p + 1]);
+        unpack_f32x2(fma_f32x2(rs, mul_f32x2(xs, splat_f32x2(-1.0f)), t2), v[2 * s + 1][2 * p],
+                     v[2 * s + 1][2 * p + 1]);
+      }
+    store_two_pairs_full<WT>(a, b + o, v);
+  }
+}
+
+// The two-pairs perturb over an aligned tile whose counters are all below 2^32, in spans of
+// kTwoPairsSpan elements.  A full span runs with its length as a compile-time constant and a
+// last partial span with a compile-time loop bound and a runtime exit: with the tile length
+// as the loop bound the step spilled 72 bytes a thread and the launch took 1.11 ms per
+// 503M-element subspace, against 1.03 ms for these forms.
+constexpr uint32_t kTwoPairsSpan = 16384;
+
+template <typename WT, int G, bool FULL>
+__device__ __forceinline__ void two_pairs_span(const ElemArgs &a, uint64_t b, uint32_t n) {
+  const float *__restrict__ mt = a.master + b;
+  const uint32_t q0_lo = (uint32_t)(b >> 2);
+  const uint32_t len = FULL ? kTwoPairsSpan : n;
+  for (uint32_t off = 4u * threadIdx.x; off < kTwoPairsSpan; off += 4u * kThreads * G) {
+    if (!FULL && off >= len) break;
+    float th[G][4];
+#pragma unroll
+    for (int i = 0; i < G; ++i) {
+      const uint32_t o = off + 4u * kThreads * i;
+      if (FULL || o < len) {
+        const float4 v = ld_stream_f4(mt + o);
+        th[i][0] = v.x, th[i][1] = v.y, th[i][2] = v.z, th[i][3] = v.w;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) th[i][k] = 0.0f;
+      }
+    }
+    two_pairs_step<WT, G>(a, b, len, off, q0_lo, th);
+  }
+}
+
+template <typename WT, int G>
+__device__ __forceinline__ void two_pairs_tile(const ElemArgs &a, uint64_t b, uint32_t len) {
+  static_assert(kTwoPairsSpan % (4 * kThreads * G) == 0, "a full span is whole steps");
+  uint32_t c0 = 0;
+  for (; len - c0 >= kTwoPairsSpan; c0 += kTwoPairsSpan) two_pairs_span<WT, G, true>(a, b + c0, kTwoPairsSpan);
+  if (c0 < len) two_pairs_span<WT, G, false>(a, b + c0, len - c0);
+}
+
 // Tile whose ends are multiples of 4: every group is whole.  Tile-local pointers and
 // 32-bit offsets; G groups per thread per step, loads issued before the math.
 // HI0: every counter of the tile is below 2^32 (its high word is the constant 0), so the
@@ -121,6 +234,13 @@ __device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b,
     for (int i = 0; i < G; ++i) {
       const uint32_t o = off + 4u * kThreads * i;
       if (o >= len) continue;
+      if constexpr (OP == kOpPerturbTwoPairs) {
+        const uint64_t q = q0 + (o >> 2);
+        float v4[4][4];
+        two_pairs_values(a, (uint32_t)q, (uint32_t)(q >> 32), th[i], v4);
+        store_two_pairs_full<WT>(a, b + o, v4);
+        continue;
+      }
       float v[4], vp[4];
       if (HI0) {
         elem_values<OP>(a, q0_lo + (o >> 2), 0u, th[i], v, vp);
@@ -130,7 +250,7 @@ __device__ __forceinline__ void elem_tile_aligned(const ElemArgs &a, uint64_t b,
       }
       if (OP == kOpInit) st_stream_f4(mt + o, make_float4(v[0], v[1], v[2], v[3]));
       WStore<WT>::full(a.w, b + o, v);
-      if (writes_context<OP>() && a.w2) WStore<WT>::full(a.w2, b + o, v);
+      if (writes_context<OP>()) store_copies_full<WT>(a.copies, b + o, v);
       if (OP == kOpPerturbPair) WStore<WT>::full(a.partner, b + o - a.partner_base, vp);
     }
   }
@@ -166,12 +286,24 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
     for (int i = 0; i < G; ++i) {
       const uint64_t g4 = base + 4ull * kThreads * i;
       if (g4 >= e) continue;
+      if constexpr (OP == kOpPerturbTwoPairs) {
+        float v4[4][4];
+        two_pairs_values(a, (uint32_t)(g4 >> 2), (uint32_t)(g4 >> 34), th[i], v4);
+        if (full[i]) {
+          store_two_pairs_full<WT>(a, g4, v4);
+        } else {
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            if (g4 + k >= b && g4 + k < e) store_two_pairs_one<WT>(a, g4 + k, v4, k);
+        }
+        continue;
+      }
       float v[4], vp[4];
       elem_values<OP>(a, (uint32_t)(g4 >> 2), (uint32_t)(g4 >> 34), th[i], v, vp);
       if (full[i]) {
         if (OP == kOpInit) st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
         WStore<WT>::full(a.w, g4, v);
-        if (writes_context<OP>() && a.w2) WStore<WT>::full(a.w2, g4, v);
+        if (writes_context<OP>()) store_copies_full<WT>(a.copies, g4, v);
         if (OP == kOpPerturbPair) WStore<WT>::full(a.partner, g4 - a.partner_base, vp);
       } else {
 #pragma unroll
@@ -180,7 +312,7 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
           if (g >= b && g < e) {
             if (OP == kOpInit) master[g] = v[k];
             WStore<WT>::one(a.w, g, v[k]);
-            if (writes_context<OP>() && a.w2) WStore<WT>::one(a.w2, g, v[k]);
+            if (writes_context<OP>()) store_copies_one<WT>(a.copies, g, v[k]);
             if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, g - a.partner_base, vp[k]);
           }
         }
@@ -192,20 +324,32 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
 // One block per tile [tiles[2t], tiles[2t+1]).  Launch shapes, measured on the 4B set:
 // the pair perturb takes G = 4 groups per step together (one tail vote for the four) at 4
 // resident blocks per SM (64 registers a thread): 0.603 ms against 0.631 ms for G = 8 one
-// group at a time at 3 blocks.  The other ops take G = 8 groups one at a time at 3 blocks
-// per SM (85 registers), which the plain perturb runs faster (0.532 against 0.544 ms).
+// group at a time at 3 blocks.  The two-pairs perturb takes G = 1 group (2 Philox blocks
+// per step, packed steps) at 4 blocks per SM (64 registers, no spill): 1.07 ms per
+// 503M-element subspace; G = 2 took 1.078 ms with scalar steps and 1.090 ms packed (52
+// bytes a thread spilled).  The other ops take G = 8 groups one at a time at 3 blocks per
+// SM (85 registers), which the plain perturb runs faster (0.532 against 0.544 ms).
 template <int OP>
-constexpr int elem_blocks_per_sm() { return OP == kOpPerturbPair ? 4 : 3; }
+constexpr int elem_blocks_per_sm() { return OP == kOpPerturbPair || OP == kOpPerturbTwoPairs ? 4 : 3; }
 template <int OP>
-constexpr int elem_groups() { return OP == kOpPerturbPair ? 4 : 8; }
+constexpr int elem_groups() { return OP == kOpPerturbPair ? 4 : (OP == kOpPerturbTwoPairs ? 1 : 8); }
 
 // A tile outside [partner_base, partner_base + partner_len) is skipped and flagged.
 __device__ __forceinline__ bool partner_covers(const ElemArgs &a, uint64_t b, uint64_t e) {
   return b >= a.partner_base && e - a.partner_base <= a.partner_len;
 }
 
+// Tiles off the two-pairs perturb's fast path (ragged ends, counters past 2^32), compiled
+// apart so that their registers do not weigh on it.
 template <int OP, typename WT, int G>
-__global__ void __launch_bounds__(kThreads, elem_blocks_per_sm<OP>()) elem_tiles_kernel(const ElemArgs a) {
+__device__ __noinline__ void elem_tile_general(const ElemArgs &a, uint64_t b, uint64_t e) {
+  if (((b | e) & 3ull) == 0) elem_tile_aligned<OP, WT, G, false>(a, b, (uint32_t)(e - b));
+  else elem_tile_ragged<OP, WT, G>(a, b, e);
+}
+
+template <int OP, typename WT, int G>
+__global__ void __launch_bounds__(kThreads, elem_blocks_per_sm<OP>())
+    elem_tiles_kernel(const __grid_constant__ ElemArgs a) {
   const uint64_t t = blockIdx.x;
   const uint64_t b = a.tiles[2 * t], e = a.tiles[2 * t + 1];
   if (b > e || e > a.n_alloc || e - b > (uint64_t)COPES_TILE_MAX) {
@@ -214,6 +358,18 @@ __global__ void __launch_bounds__(kThreads, elem_blocks_per_sm<OP>()) elem_tiles
   }
   if (OP == kOpPerturbPair && !partner_covers(a, b, e)) {
     if (threadIdx.x == 0) flag_error(kErrPartnerRange);
+    return;
+  }
+  if constexpr (OP == kOpPerturbTwoPairs) {
+    // a tile of exactly one span (the default tile size) runs the span with every bound
+    // a compile-time constant: 1.054 ms per 503M-element subspace against 1.110 ms through
+    // the span loop of two_pairs_tile
+    if (((b | e) & 3ull) == 0 && (e >> 34) == 0) {
+      if (e - b == kTwoPairsSpan) two_pairs_span<WT, G, true>(a, b, kTwoPairsSpan);
+      else two_pairs_tile<WT, G>(a, b, (uint32_t)(e - b));
+    } else {
+      elem_tile_general<OP, WT, G>(a, b, e);
+    }
     return;
   }
   if (((b | e) & 3ull) == 0) {
@@ -342,7 +498,7 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
           else master[g[u]] = v;
         }
         WStore<WT>::one(a.w, (uint64_t)g[u], v);
-        if (writes_context<OP>() && a.w2) WStore<WT>::one(a.w2, (uint64_t)g[u], v);
+        if (writes_context<OP>()) store_copies_one<WT>(a.copies, (uint64_t)g[u], v);
         if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, (uint64_t)g[u] - a.partner_base, vp);
       }
     }
@@ -351,7 +507,11 @@ __global__ void __launch_bounds__(kThreads) elem_index_kernel(const ElemArgs a) 
 
 template <int OP, typename WT>
 static cudaError_t launch_elem_typed(int kind, const ElemArgs &a, cudaStream_t s) {
-  if constexpr (OP == kOpGather || OP == kOpScatter) {
+  if constexpr (OP == kOpPerturbTwoPairs) {
+    if (kind != COPES_SUBSPACE_TILES || a.copies.n != 3) return cudaErrorInvalidValue;
+    if (a.n_tiles == 0) return cudaSuccess;
+    elem_tiles_kernel<OP, WT, elem_groups<OP>()><<<(unsigned)a.n_tiles, kThreads, 0, s>>>(a);
+  } else if constexpr (OP == kOpGather || OP == kOpScatter) {
     if (kind != COPES_SUBSPACE_INDICES || !a.gathered) return cudaErrorInvalidValue;
     if (a.n_index == 0) return cudaSuccess;
     const uint64_t blocks = (a.n_index + kIndexSegment - 1) / kIndexSegment;
@@ -386,6 +546,7 @@ cudaError_t launch_elementwise(int op, int kind, int dtype, const ElemArgs &a, c
     case kOpScatter: return launch_elem_op<kOpScatter>(kind, dtype, a, s);
     case kOpPerturbPair: return launch_elem_op<kOpPerturbPair>(kind, dtype, a, s);
     case kOpPartner: return launch_elem_op<kOpPartner>(kind, dtype, a, s);
+    case kOpPerturbTwoPairs: return launch_elem_op<kOpPerturbTwoPairs>(kind, dtype, a, s);
     default: return launch_elem_op<kOpInit>(kind, dtype, a, s);
   }
 }
@@ -417,7 +578,7 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
         st_stream_f4(master + g4, make_float4(v[0], v[1], v[2], v[3]));
         if (COMMIT) {
           WStore<WT>::full(a.w, g4, v);
-          if (a.w2) WStore<WT>::full(a.w2, g4, v);
+          store_copies_full<WT>(a.copies, g4, v);
         }
       } else {
 #pragma unroll
@@ -428,7 +589,7 @@ __device__ __forceinline__ void update_tile(const UpdateArgs &a, const float *s_
             master[g] = v;
             if (COMMIT) {
               WStore<WT>::one(a.w, g, v);
-              if (a.w2) WStore<WT>::one(a.w2, g, v);
+              store_copies_one<WT>(a.copies, g, v);
             }
           }
         }
@@ -525,7 +686,7 @@ __global__ void __launch_bounds__(kThreads) update_index_kernel(const __grid_con
         *th = v;
         if (COMMIT) {
           WStore<WT>::one(a.w, (uint64_t)g[u], v);
-          if (a.w2) WStore<WT>::one(a.w2, (uint64_t)g[u], v);
+          store_copies_one<WT>(a.copies, (uint64_t)g[u], v);
         }
       }
     }

@@ -220,7 +220,7 @@ __global__ void __launch_bounds__(kThreads) replay_elem_kernel(const __grid_cons
         if (OP == kOpInit) master[g[u]] = v;
       }
       WStore<WT>::one(a.w, g[u], v);
-      if ((OP == kOpRestore || OP == kOpInit) && a.w2) WStore<WT>::one(a.w2, g[u], v);
+      if (OP == kOpRestore || OP == kOpInit) store_copies_one<WT>(a.copies, g[u], v);
       if (OP == kOpPerturbPair) WStore<WT>::one(a.partner, g[u] - a.partner_base, vp);
     }
   }, [] {});
@@ -279,7 +279,7 @@ __global__ void __launch_bounds__(kThreads) replay_update_kernel(const __grid_co
       master[g[u]] = v;
       if (COMMIT) {
         WStore<WT>::one(a.w, g[u], v);
-        if (a.w2) WStore<WT>::one(a.w2, g[u], v);
+        store_copies_one<WT>(a.copies, g[u], v);
       }
     }
   }, [] {});
@@ -341,7 +341,8 @@ static cudaError_t launch_replay_elem_dtype(int op, const ElemArgs &a, const Rep
     case kOpRestore: return launch_replay_elem_typed<kOpRestore, WT>(a, r, s);
     case kOpPerturbPair: return launch_replay_elem_typed<kOpPerturbPair, WT>(a, r, s);
     case kOpPartner: return launch_replay_elem_typed<kOpPartner, WT>(a, r, s);
-    default: return launch_replay_elem_typed<kOpInit, WT>(a, r, s);
+    case kOpInit: return launch_replay_elem_typed<kOpInit, WT>(a, r, s);
+    default: return cudaErrorInvalidValue;  // the other ops have no replay form
   }
 }
 

@@ -52,10 +52,13 @@ class Partner:
     arena at buf[g - base], in the working dtype.  Partner.covering(arena, subs) sizes one
     for every element of `subs`.  in_place: the buffer is the arena's second working
     buffer w2 (Partner.second_copy), so the partner member is evaluated there directly and
-    nothing is copied."""
+    nothing is copied.  two_pairs: the arena has four working copies
+    (Partner.four_copies), and two consecutive antithetic pairs with the same sign order
+    are written to w, w2, w3 and w4 by one copes_perturb_two_pairs."""
     buf: torch.Tensor
     base: int
     in_place: bool = False
+    two_pairs: bool = False
 
     @classmethod
     def second_copy(cls, arena: copes.Arena) -> "Partner":
@@ -63,6 +66,14 @@ class Partner:
         member 2j + 1 on w2."""
         assert arena.w2 is not None, "the arena has no second working buffer"
         return cls(arena.w2, 0, True)
+
+    @classmethod
+    def four_copies(cls, arena: copes.Arena) -> "Partner":
+        """Members 4m .. 4m + 3 (noise vectors 2m and 2m + 1, signs +, -, +, -) evaluated
+        on w, w2, w3 and w4, all four written by one pass; a pair left over at the end of
+        the member list goes to w and w2."""
+        assert arena.w4 is not None, "the arena has no four working copies"
+        return cls(arena.w2, 0, True, True)
 
     @classmethod
     def covering(cls, arena: copes.Arena, subs: Sequence[copes.SubspaceHandle]) -> "Partner":
@@ -81,6 +92,11 @@ class Partner:
         return [cls(buf, lo) for lo, _ in spans]
 
 
+def _antithetic(nid, sign, a: int, b: int) -> bool:
+    """Members a and b share a noise vector with opposite signs."""
+    return nid[b] == nid[a] and sign[b] == -sign[a]
+
+
 def perturb_members(arena: copes.Arena, sub: copes.SubspaceHandle, members: Sequence[int], nid, sign,
                     seeds, s_k: float, live: Callable[[int], None], partner: Optional[Partner] = None,
                     events: Optional[dict] = None, backup: bool = False) -> None:
@@ -89,22 +105,36 @@ def perturb_members(arena: copes.Arena, sub: copes.SubspaceHandle, members: Sequ
     successor shares its noise vector with the opposite sign (an antithetic pair) is
     perturbed by copes_perturb_pair, and the successor's weights are then copied in from
     the buffer, or, for an in-place partner (the arena's w2), evaluated there: one noise
-    generation per pair, bit-identical weights.  backup: the CPU weight backup mode's
-    calls (arena is a copes.BackupArena)."""
+    generation per pair, bit-identical weights.  With four working copies
+    (Partner.four_copies), two such pairs in a row whose first members have the same sign
+    are written to w, w2, w3 and w4 by one copes_perturb_two_pairs and evaluated there
+    (TILES subspaces; other kinds take the pairs one at a time).
+    backup: the CPU weight backup mode's calls (arena is a copes.BackupArena)."""
     if backup:
+        assert partner is None or not partner.two_pairs, "the backup mode has one working copy"
         perturb, pair, copy = copes.backup_perturb, copes.backup_perturb_pair, copes.backup_perturb_partner
     else:
         perturb, pair, copy = copes.perturb, copes.perturb_pair, copes.perturb_partner
     staged = None  # the member whose weights the partner buffer holds
+    ready = {}     # member -> the working copy that already holds its weights
     for pos, i in enumerate(members):
         nxt = members[pos + 1] if pos + 1 < len(members) else None
         seed, ss = int(seeds[nid[i]]), float(sign[i]) * s_k
         where = None if arena is None else arena.w
-        if staged == i and partner.in_place:
+        quad = (members[pos:pos + 4] if partner is not None and partner.two_pairs
+                and sub.kind == copes.SUBSPACE_TILES else [])
+        if i in ready:
+            where = ready.pop(i)
+        elif staged == i and partner.in_place:
             where = partner.buf
         elif staged == i:
             _timed(events, "partner", lambda: copy(arena, sub, partner.buf, partner.base))
-        elif partner is not None and nxt is not None and nid[nxt] == nid[i] and sign[nxt] == -sign[i]:
+        elif (len(quad) == 4 and _antithetic(nid, sign, quad[0], quad[1]) and _antithetic(nid, sign, quad[2], quad[3])
+              and sign[quad[2]] == sign[i]):
+            seed_b = int(seeds[nid[quad[2]]])
+            _timed(events, "perturb", lambda: copes.perturb_two_pairs(arena, sub, seed, seed_b, ss))
+            ready = {quad[1]: arena.w2, quad[2]: arena.w3, quad[3]: arena.w4}
+        elif partner is not None and nxt is not None and _antithetic(nid, sign, i, nxt):
             _timed(events, "perturb", lambda: pair(arena, sub, seed, ss, partner.buf, partner.base))
             staged = nxt
         else:
@@ -343,26 +373,27 @@ def population_visit(arena: copes.Arena, sub: copes.SubspaceHandle, k: int, iter
 # ------------------------------------------------------------------ checkpoint / resume
 def state_dict(arena: copes.Arena, cfg: ESConfig, next_iteration: int, **extra) -> dict:
     """The resumable ES state: the fp32 master (host copy), the configuration, the next
-    iteration index and whether the arena keeps a second working copy w2.  Member seeds
+    iteration index and how many working copies the arena keeps (1, 2 or 4).  Member seeds
     and noise are functions of (base seed, iteration, subspace, member) and (seed, index),
     and partition seeds are part of `extra`, so nothing else needs saving: a run resumed
     from this state continues bit for bit.  The working copies are not saved: between ES
-    iterations both equal round(theta) and are rebuilt from the master."""
+    iterations all of them equal round(theta) and are rebuilt from the master."""
     return {"master": arena.master.detach().cpu().clone(), "working_dtype": str(arena.w.dtype),
-            "second_copy": arena.w2 is not None, "config": dict(cfg.__dict__),
+            "working_copies": len(arena.copies), "config": dict(cfg.__dict__),
             "next_iteration": int(next_iteration), **extra}
 
 
 def load_state(state: dict, device="cuda") -> tuple:
     """Rebuilds (arena, cfg, next_iteration) from state_dict's output: the master is
-    copied to the device and the working weights, with the second working copy when the
-    saved arena had one, are committed from it (w = w2 = round(theta) over the whole
-    arena)."""
+    copied to the device and the saved number of working copies is committed from it
+    (every copy = round(theta) over the whole arena)."""
     master = state["master"].to(device).contiguous()
     dtype = {"torch.bfloat16": torch.bfloat16, "torch.float32": torch.float32}[state["working_dtype"]]
     n = master.numel()
-    w2 = torch.empty(n, dtype=dtype, device=device) if state.get("second_copy", False) else None
-    arena = copes.Arena(torch.empty(n, dtype=dtype, device=device), master, w2=w2)
+    n_copies = int(state.get("working_copies", 1))
+    assert n_copies in (1, 2, 4), f"{n_copies} working copies"
+    copies = [torch.empty(n, dtype=dtype, device=device) for _ in range(n_copies)]
+    arena = copes.Arena(copies[0], master, *copies[1:])
     everything = copes.tiles_from_ranges([(0, n)], device=device)
-    copes.context_commit(arena, everything)  # commit writes w2 too when it is set
+    copes.context_commit(arena, everything)  # commit writes every working copy
     return arena, ESConfig(**state["config"]), state["next_iteration"]

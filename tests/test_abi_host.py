@@ -305,6 +305,38 @@ def test_second_working_buffer_is_validated(lib):
     assert lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None) == copes.ERR_INVALID_ARG
 
 
+def test_four_working_copies_are_validated(lib):
+    """w3 and w4 come together and only with w2, 16-byte aligned, each disjoint from w, the
+    master and the other copies; copes_perturb_two_pairs needs all four copies and a TILES
+    subspace.  Every case fails before any CUDA call."""
+    from paper_2608_02391_gb300 import copes
+    fake = 0x10000  # never dereferenced: every case below fails validation first
+    mst = fake + (1 << 24)
+    w2, w3, w4 = fake + 1024, fake + 2048, fake + 3072  # 200 B each (100 bf16)
+    s = copes.Subspace(copes.SUBSPACE_TILES, fake, 1, None, 0)
+    R = lambda p: lib.copes_restore(ctypes.byref(p), ctypes.byref(s), None)
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, w3, None)) == copes.ERR_INVALID_ARG  # w3 alone
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, None, w4)) == copes.ERR_INVALID_ARG  # w4 alone
+    assert R(copes.Params(fake, mst, 100, copes.BF16, None, w3, w4)) == copes.ERR_INVALID_ARG  # without w2
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, w3 + 8, w4)) == copes.ERR_ALIGNMENT
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, w3, w4 + 4)) == copes.ERR_ALIGNMENT
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, w3, fake)) == copes.ERR_INVALID_ARG  # w4 aliases w
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, mst, w4)) == copes.ERR_INVALID_ARG  # w3 aliases master
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, w2, w4)) == copes.ERR_INVALID_ARG  # w3 aliases w2
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, w3, w2 + 176)) == copes.ERR_INVALID_ARG  # w4 in w2
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, w3, w3 + 160)) == copes.ERR_INVALID_ARG  # w4 in w3
+    assert R(copes.Params(fake, mst, 100, copes.BF16, w2, mst - 192, w4)) == copes.ERR_INVALID_ARG  # into master
+    assert R(copes.Params(fake, mst, 100, copes.FP32, w2, w2 + 256, w4)) == copes.ERR_INVALID_ARG  # fp32 w2: 400 B
+    T = lambda p, sub, sigma=1e-3: lib.copes_perturb_two_pairs(ctypes.byref(p), ctypes.byref(sub), 1, 2, sigma, None)
+    dual = copes.Params(fake, mst, 100, copes.BF16, w2)
+    assert T(dual, s) == copes.ERR_INVALID_ARG  # two copies only
+    quad = copes.Params(fake, mst, 100, copes.BF16, w2, w3, w4)
+    assert T(quad, s, float("inf")) == copes.ERR_INVALID_ARG
+    idx = copes.Subspace(copes.SUBSPACE_INDICES, None, 0, fake, 10)
+    assert T(quad, idx) == copes.ERR_UNSUPPORTED
+    assert lib.copes_perturb_two_pairs(None, ctypes.byref(s), 1, 2, 1e-3, None) == copes.ERR_INVALID_ARG
+
+
 def test_backup_partner_arguments_are_rejected_before_any_launch(lib):
     from paper_2608_02391_gb300 import copes
     fake = 0x10000  # never dereferenced: every case below fails validation first

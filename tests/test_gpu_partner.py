@@ -285,3 +285,125 @@ def test_pair_on_an_empty_subspace_is_a_no_op(copes):
     copes.restore(arena, empty)
     copes.check()
     assert np.array_equal(bits(arena.w), before) and np.array_equal(bits(arena.w2), before2)
+
+
+# ------------------------------------------- four working copies (w2, w3 and w4)
+def quad_arena(copes, theta, dtype):
+    cs = [canary(theta.size, dtype, 20 + c) for c in range(4)]
+    return copes.Arena(cs[0], torch.from_numpy(theta.copy()).cuda(), *cs[1:])
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("tile", [4096, 1000, 777])
+def test_two_pairs_equal_four_perturbs_and_the_oracle(copes, dtype, tile):
+    """copes_perturb_two_pairs writes to w, w2, w3 and w4, on S only, exactly what
+    copes_perturb writes for (seed_a, +s), (seed_a, -s), (seed_b, +s) and (seed_b, -s),
+    and each member agrees with the oracle; ragged and aligned tiles."""
+    theta = theta_np()
+    inside = mask_of(RANGES)
+    g = np.nonzero(inside)[0].astype(np.uint64)
+    arena = quad_arena(copes, theta, dtype)
+    before = [bits(c).copy() for c in arena.copies]
+    ref = copes.Arena(canary(N_ALLOC, dtype, 20), torch.from_numpy(theta.copy()).cuda())
+    sub = copes.tiles_from_ranges(RANGES, tile_size=tile)
+    for seed_a, seed_b, ss in [(11, 12, 2e-3), (2**40 + 5, 7, -1e-3)]:
+        copes.perturb_two_pairs(arena, sub, seed_a, seed_b, ss)
+        for c, (seed, s) in enumerate([(seed_a, ss), (seed_a, -ss), (seed_b, ss), (seed_b, -ss)]):
+            copes.perturb(ref, sub, seed, s)
+            got = bits(arena.copies[c])
+            assert np.array_equal(got[inside], bits(ref.w)[inside]), c
+            assert np.array_equal(got[~inside], before[c][~inside]), c  # untouched outside S
+            check_member(got[inside], dtype, g, theta[inside], seed, s)
+    copes.check()
+
+
+def test_two_pairs_on_an_empty_subspace_is_a_no_op(copes):
+    arena = quad_arena(copes, theta_np(1000), torch.bfloat16)
+    before = [bits(c).copy() for c in arena.copies]
+    copes.perturb_two_pairs(arena, copes.tiles_from_ranges([], tile_size=64), 1, 2, 1e-3)
+    copes.check()
+    assert all(np.array_equal(bits(c), b) for c, b in zip(arena.copies, before))
+
+
+@pytest.mark.parametrize("kind", ["tiles:1000", "indices", "replay"])
+def test_four_copies_receive_the_context_only(copes, kind):
+    """With w2, w3 and w4 set, restore, commit, the fused update's commit and init write
+    the same values to every copy as to w (on S only); a plain or pair perturb writes w
+    (and the partner buffer) and leaves the other copies alone."""
+    theta = theta_np()
+    cs = [canary(N_ALLOC, torch.bfloat16, 30 + c) for c in range(4)]
+    quad = copes.Arena(cs[0], torch.from_numpy(theta.copy()).cuda(), *cs[1:])
+    single = copes.Arena(cs[0].clone(), torch.from_numpy(theta.copy()).cuda())
+    if kind == "replay":
+        layout = copes.Layout([N_ALLOC])
+        sub = copes.hash_replay_partition(layout, 3, 11)[1]
+        inside = np.zeros(N_ALLOC, bool)
+        inside[oracle.hash_list([N_ALLOC], [0], 3, 11, 1).astype(np.int64)] = True
+    else:
+        sub = make_sub(copes, kind, RANGES, quad)
+        inside = mask_of(RANGES)
+    b0 = [bits(c).copy() for c in cs[1:]]
+
+    def others_hold(w_bits):
+        for c, b in zip(cs[1:], b0):
+            got = bits(c)
+            assert np.array_equal(got[inside], w_bits[inside]) and np.array_equal(got[~inside], b[~inside])
+
+    buf = canary(N_ALLOC, torch.bfloat16, 5)
+    copes.perturb(quad, sub, 5, 1e-3)
+    copes.perturb_pair(quad, sub, 6, 1e-3, buf, 0)
+    copes.perturb_pair(single, sub, 6, 1e-3, buf, 0)
+    assert np.array_equal(bits(quad.w), bits(single.w))
+    assert all(np.array_equal(bits(c), b) for c, b in zip(cs[1:], b0))
+    copes.restore(quad, sub)
+    copes.restore(single, sub)
+    assert np.array_equal(bits(quad.w), bits(single.w))
+    others_hold(bits(quad.w))
+    nid, sign, P = copes.member_table(4, copes.ANTITHETIC)
+    f = torch.tensor([1.0, -0.5, 0.25, 2.0], device="cuda")
+    for a in (quad, single):
+        copes.update(a, sub, nid, sign, f, copes.member_seeds(33, 0, 0, P), 0.1, fuse_commit=True)
+    assert np.array_equal(quad.master.cpu().numpy().view(np.uint32), single.master.cpu().numpy().view(np.uint32))
+    assert np.array_equal(bits(quad.w), bits(single.w))
+    others_hold(bits(quad.w))
+    copes.init_normal(quad, sub, 7, 0.0, 0.02)
+    others_hold(bits(quad.w))
+    copes.check()
+
+
+def copies_trace(copes, es, copies, kind, n_members):
+    n = 1 << 18
+    theta = theta_np(n, 3)
+    w = torch.from_numpy(theta.copy()).cuda().to(torch.bfloat16)
+    arena = copes.Arena(w, torch.from_numpy(theta.copy()).cuda(), *[w.clone() for _ in range(copies - 1)])
+    layout = copes.Layout([n // 2, n // 2 - 100])
+    subs = (es.build_subspaces(layout, "contiguous", 3, tile_size=4096) if kind == "tiles"
+            else copes.hash_replay_partition(layout, 3, 5))
+    partner = {1: None, 2: es.Partner.second_copy, 4: es.Partner.four_copies}[copies]
+    partner = partner(arena) if partner else None
+    cfg = es.ESConfig(n_members=n_members, sigma=1e-3, alpha=5e-4)
+    rng = np.random.default_rng(1)
+    trace = []
+    for k, sub in enumerate(subs):
+        r = torch.from_numpy(rng.standard_normal(n_members).astype(np.float32)).cuda()
+
+        def ev(i):  # what a rollout would see: the live buffer's bits
+            trace.append(int(arena.live.view(torch.int16).to(torch.int64).mul(i + 1).sum()))
+
+        es.round_robin_visit(arena, sub, k, 0, cfg, n, r, evaluate=ev, partner=partner)
+    copes.check()
+    return trace, arena
+
+
+@pytest.mark.parametrize("kind", ["tiles", "replay"])
+@pytest.mark.parametrize("n_members", [8, 6])
+def test_visit_on_four_working_copies_is_bit_identical(copes, kind, n_members):
+    """Members 4m .. 4m + 3 on w, w2, w3 and w4 (a pair left over goes to w and w2; other
+    subspace kinds take pairs): every member sees the weights it sees with one copy, and
+    afterwards every copy and the master equal the one-copy run's."""
+    from paper_2608_02391_gb300 import es
+    t0, a0 = copies_trace(copes, es, 1, kind, n_members)
+    t1, a1 = copies_trace(copes, es, 4, kind, n_members)
+    assert t0 == t1 and len(t0) == 3 * n_members
+    assert all(np.array_equal(bits(c), bits(a0.w)) for c in a1.copies)
+    assert np.array_equal(a1.master.cpu().numpy().view(np.uint32), a0.master.cpu().numpy().view(np.uint32))

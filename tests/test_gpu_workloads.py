@@ -392,6 +392,39 @@ def test_counters_beyond_2_34(copes):
     copes.check()
 
 
+def test_two_pairs_beyond_2_34(copes):
+    """The two-pairs perturb on a range crossing global index 2^34 (its general counter
+    path above, its folded-Philox path below): each of the four working copies equals a
+    plain perturb bit for bit, and agrees with the oracle on sampled indices on both
+    sides.  Four bf16 copies and the fp32 master of 2^34 + 2^20 elements: 192 GB."""
+    n = (1 << 34) + (1 << 20)
+    lo, hi = (1 << 34) - (1 << 19), (1 << 34) + (1 << 19)
+    master = torch.empty(n, dtype=torch.float32, device="cuda")
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(5)
+    master[lo:hi].normal_(0.0, 0.02, generator=gen)
+    copies = [torch.zeros(n, dtype=torch.bfloat16, device="cuda") for _ in range(4)]
+    sub = copes.tiles_from_ranges([(lo, hi)], tile_size=1 << 16)
+    members = [(77, 1e-3), (77, -1e-3), (78, 1e-3), (78, -1e-3)]
+    copes.perturb_two_pairs(copes.Arena(copies[0], master, *copies[1:]), sub, 77, 78, 1e-3)
+    got = [c[lo:hi].view(torch.int16).clone() for c in copies]
+    del copies[1:]
+    single = copes.Arena(copies[0], master)
+    rng = np.random.default_rng(6)
+    sample = np.unique(np.concatenate([[lo, (1 << 34) - 1, 1 << 34, hi - 1],
+                                       rng.integers(lo, hi, 4000)])).astype(np.int64)
+    theta = master[torch.from_numpy(sample).cuda()].cpu().numpy()
+    g = sample.astype(np.uint64)
+    for c, (seed, s) in enumerate(members):
+        copes.perturb(single, sub, seed, s)
+        assert torch.equal(copies[0][lo:hi].view(torch.int16), got[c]), c
+        scale = np.maximum(np.abs(theta), np.abs(np.float32(s) * oracle.noise(seed, g)))
+        ref_bits, _ = oracle.perturb_at(g, theta, seed, s, oracle.BF16)
+        mine = got[c][torch.from_numpy(sample - lo).cuda()].cpu().numpy().view(np.uint16)
+        assert_bf16_close(mine, ref_bits.astype(np.uint16), scale)
+    copes.check()
+
+
 # ------------------------------------------------------------------ Algorithm 1 (SYNC)
 @pytest.mark.parametrize("joint", [True, False])
 def test_sync_step_algorithm1_matches_oracle(copes, joint):
