@@ -57,17 +57,22 @@ sys.path.insert(0, ROOT)
 METRIC = "ES-iteration params/s and HBM GB/s at 4B bf16 (N=32), % of roofline on 1 GB300"
 FALLBACK_HBM_GBS = 6800.0
 
-# ncu DRAM bytes per element of the dominant kernel (the pair perturb, or the plain perturb
-# under --weights single; bf16) from one capture each; a figure is dropped (traffic = null)
-# when the tile kernels' sources (source_sha) no longer match the hash it was taken on.
-# The pair perturb's figure comes from subspaces of 2^28 parameters, where the writes still
-# in L2 when the kernel ends are about 2% of its traffic.
+# ncu DRAM bytes per element of the dominant kernel (the two-pairs perturb, the pair
+# perturb under --weights dual or partner, the plain perturb under --weights single; bf16)
+# from one capture each; a figure is dropped (traffic = null) when the tile kernels'
+# sources (source_sha) no longer match the hash it was taken on.  The figures come from
+# subspaces of 2^28 parameters, where the writes still in L2 when the kernel ends are about
+# 2% of its traffic.
 NCU_TRAFFIC = {
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "dc47c2eb721dab12",
-                     "bytes_per_elem": 7.827, "capture": "profiles/perturb_pair_4b_slice.md",
-                     "case": "two 2^28-parameter subspaces (--case 4b-slice-big)"},
-    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "35ede1dfa8ae5289",
-                "bytes_per_elem": 5.413, "capture": "profiles/perturb_4b_slice.md"},
+    "perturb_two_pairs": {"kernel": "elem_tiles_kernel<perturb_two_pairs,bf16>", "source_sha": "242a48997503aee4",
+                          "bytes_per_elem": 11.781, "capture": "profiles/perturb_two_pairs_4b_slice.md",
+                          "case": "two 2^28-parameter subspaces (--case 4b-slice-big)"},
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "242a48997503aee4",
+                     "bytes_per_elem": 7.826, "capture": "profiles/perturb_pair_4b_slice.md",
+                     "case": "two 2^28-parameter subspaces (--case 4b-slice-big --weights dual)"},
+    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "242a48997503aee4",
+                "bytes_per_elem": 5.862, "capture": "profiles/perturb_4b_slice.md",
+                "case": "two 2^28-parameter subspaces (--case 4b-slice-big --weights single)"},
 }
 
 
@@ -91,8 +96,9 @@ def parse():
     ap.add_argument("--cpu-sample", type=int, default=1 << 20,
                     help="parameters of the oracle's timed CPU sample")
     ap.add_argument("--weights", default=None, choices=["quad", "dual", "partner", "single"],
-                    help="quad (default for tile subspaces): four working-weight copies, two antithetic "
-                         "pairs written by one pass; dual (default for the hash and backup cases): two "
+                    help="quad (default for the round-robin tile cases): four working-weight copies, two "
+                         "antithetic pairs written by one pass; dual (default for the hash, backup and sync "
+                         "cases): two "
                          "working-weight copies, antithetic members 2j on w and 2j+1 on w2 (one pair "
                          "perturb per pair; the backup case keeps one copy and a partner buffer); partner: "
                          "one copy, member 2j+1 copied in from a partner buffer; single: one copy, every "
@@ -442,8 +448,9 @@ def main():
     args = parse()
     from paper_2608_02391_gb300 import workloads
     wl = workloads.workload({"4b-backup": "4b", "4b-sync": "4b", "4b-backup-slice": "4b-slice"}.get(args.case, args.case))
-    if args.weights is None:
-        args.weights = "dual" if wl.mode == "hash" or args.case in ("4b-backup", "4b-backup-slice") else "quad"
+    if args.weights is None:  # four copies pay off where a restore serves many members
+        args.weights = "quad" if wl.mode != "hash" and args.case not in ("4b-backup", "4b-backup-slice",
+                                                                          "4b-sync") else "dual"
     if args.impl == "reference":
         return run_reference(args, wl)
 

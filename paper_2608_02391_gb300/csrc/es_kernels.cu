@@ -339,14 +339,6 @@ __device__ __forceinline__ bool partner_covers(const ElemArgs &a, uint64_t b, ui
   return b >= a.partner_base && e - a.partner_base <= a.partner_len;
 }
 
-// Tiles off the two-pairs perturb's fast path (ragged ends, counters past 2^32), compiled
-// apart so that their registers do not weigh on it.
-template <int OP, typename WT, int G>
-__device__ __noinline__ void elem_tile_general(const ElemArgs &a, uint64_t b, uint64_t e) {
-  if (((b | e) & 3ull) == 0) elem_tile_aligned<OP, WT, G, false>(a, b, (uint32_t)(e - b));
-  else elem_tile_ragged<OP, WT, G>(a, b, e);
-}
-
 template <int OP, typename WT, int G>
 __global__ void __launch_bounds__(kThreads, elem_blocks_per_sm<OP>())
     elem_tiles_kernel(const __grid_constant__ ElemArgs a) {
@@ -367,8 +359,10 @@ __global__ void __launch_bounds__(kThreads, elem_blocks_per_sm<OP>())
     if (((b | e) & 3ull) == 0 && (e >> 34) == 0) {
       if (e - b == kTwoPairsSpan) two_pairs_span<WT, G, true>(a, b, kTwoPairsSpan);
       else two_pairs_tile<WT, G>(a, b, (uint32_t)(e - b));
+    } else if (((b | e) & 3ull) == 0) {
+      elem_tile_aligned<OP, WT, G, false>(a, b, (uint32_t)(e - b));
     } else {
-      elem_tile_general<OP, WT, G>(a, b, e);
+      elem_tile_ragged<OP, WT, G>(a, b, e);
     }
     return;
   }
