@@ -64,13 +64,13 @@ FALLBACK_HBM_GBS = 6800.0
 # subspaces of 2^28 parameters, where the writes still in L2 when the kernel ends are about
 # 2% of its traffic.
 NCU_TRAFFIC = {
-    "perturb_two_pairs": {"kernel": "elem_tiles_kernel<perturb_two_pairs,bf16>", "source_sha": "242a48997503aee4",
-                          "bytes_per_elem": 11.781, "capture": "profiles/perturb_two_pairs_4b_slice.md",
+    "perturb_two_pairs": {"kernel": "elem_tiles_kernel<perturb_two_pairs,bf16>", "source_sha": "6adf05ff51bf21e3",
+                          "bytes_per_elem": 11.782, "capture": "profiles/perturb_two_pairs_4b_slice.md",
                           "case": "two 2^28-parameter subspaces (--case 4b-slice-big)"},
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "242a48997503aee4",
-                     "bytes_per_elem": 7.826, "capture": "profiles/perturb_pair_4b_slice.md",
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "6adf05ff51bf21e3",
+                     "bytes_per_elem": 7.827, "capture": "profiles/perturb_pair_4b_slice.md",
                      "case": "two 2^28-parameter subspaces (--case 4b-slice-big --weights dual)"},
-    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "242a48997503aee4",
+    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "6adf05ff51bf21e3",
                 "bytes_per_elem": 5.862, "capture": "profiles/perturb_4b_slice.md",
                 "case": "two 2^28-parameter subspaces (--case 4b-slice-big --weights single)"},
 }

@@ -2,7 +2,8 @@
  * device memory from the CUDA runtime (cudaMalloc), every step of the visit a copes_*
  * call -- copes_subspace_build, N x copes_perturb, copes_restore, copes_shape_fitness,
  * copes_update without the fused commit, then copes_context_commit (Sec. 3.2, Eq. 8,
- * Eq. 5, Eq. 13).  Inputs come from a host generator; every input and output is dumped
+ * Eq. 5, Eq. 13).  Before the restore it also runs copes_perturb_two_pairs on four working
+ * copies (members 0 .. 3 in one pass, Eq. 8).  Inputs come from a host generator; every input and output is dumped
  * as a raw little-endian file into the directory argv[1], and the run's scalars are
  * printed one per line, for tests/test_c_abi_gpu.py to check against the oracle.
  * Exit status: 0 on success, 2 when a copes_* call fails, 3 when a CUDA call fails. */
@@ -151,6 +152,22 @@ int main(int argc, char **argv) {
     for (uint64_t g = 0; g < n; ++g) r += c[g] * (double)bf16_to_float(wh[g]);
     rewards[i] = (float)r;
   }
+  /* members 0 .. 3 (noise vectors 0 and 1, signs +, -, +, -) in one pass into four
+   * working copies, whose context is committed first */
+  void *wc[3];
+  for (int c = 0; c < 3; ++c) CU(cudaMalloc(&wc[c], n * sizeof(uint16_t)));
+  const copes_params p4 = {w, master, n, COPES_BF16, wc[0], wc[1], wc[2]};
+  CK(copes_context_commit(&p4, &all, s));
+  CK(copes_perturb_two_pairs(&p4, &S, seeds[nid[0]], seeds[nid[2]], (float)sign[0] * sigma, s));
+  for (int c = 0; c < 4; ++c) {
+    char name[64];
+    snprintf(name, sizeof name, "w_two_pairs%d.bin", c);
+    CU(cudaMemcpyAsync(wh, c ? wc[c - 1] : w, n * sizeof(uint16_t), cudaMemcpyDeviceToHost, s));
+    CU(cudaStreamSynchronize(s));
+    if (dump(dir, name, wh, n * sizeof(uint16_t))) return 1;
+  }
+  for (int c = 0; c < 3; ++c) CU(cudaFree(wc[c]));
+
   CK(copes_restore(&p, &S, s));
   CU(cudaMemcpyAsync(wh, w, n * sizeof(uint16_t), cudaMemcpyDeviceToHost, s));
   CU(cudaStreamSynchronize(s));

@@ -1,8 +1,9 @@
 """One ES visit driven from plain C: tests/c_abi_visit.c allocates with cudaMalloc and
-calls only include/copes.h -- copes_subspace_build, N x copes_perturb, copes_restore,
-copes_shape_fitness, copes_update (fuse_commit = 0) and copes_context_commit -- on a
-3-tensor layout; its dumps are checked here against the oracle (Sec. 3.2, Eq. 8, Eq. 5,
-Eq. 13) at the tolerances of tests/tolerances.py."""
+calls only include/copes.h -- copes_subspace_build, N x copes_perturb,
+copes_perturb_two_pairs on four working copies, copes_restore, copes_shape_fitness,
+copes_update (fuse_commit = 0) and copes_context_commit -- on a 3-tensor layout; its
+dumps are checked here against the oracle (Sec. 3.2, Eq. 8, Eq. 5, Eq. 13) at the
+tolerances of tests/tolerances.py."""
 import os
 import shutil
 import subprocess
@@ -48,7 +49,8 @@ def visit(tmp_path_factory):
     d = {name: load(name + ".bin", dt) for name, dt in [
         ("theta", np.float32), ("rewards", np.float32), ("fitness", np.float32), ("master_after", np.float32),
         ("w_member0", np.uint16), ("w_member1", np.uint16), ("w_restored", np.uint16),
-        ("w_before_commit", np.uint16), ("w_after", np.uint16), ("tiles", np.uint64)]}
+        ("w_before_commit", np.uint16), ("w_after", np.uint16), ("tiles", np.uint64),
+        *[(f"w_two_pairs{c}", np.uint16) for c in range(4)]]}
     d.update(n=n, P=int(lines["P"]), seeds=np.array(lines["seeds"].split(), dtype=np.uint64),
              coef=np.float32(float(lines["coef"])))
     assert all(d[x].size == n for x in ("theta", "master_after", "w_after"))
@@ -114,3 +116,24 @@ def test_shaping_update_and_commit_from_c(visit):
     assert np.array_equal(visit["w_before_commit"], visit["w_restored"])
     # the commit published round(theta) of the new master
     assert np.array_equal(visit["w_after"], oracle.bf16_bits_array(after))
+
+
+def test_two_pairs_from_c(visit):
+    """copes_perturb_two_pairs from C: copies 0 and 1 equal the plain perturbs of members 0
+    and 1 bit for bit, copies 2 and 3 (members 2 and 3) agree with the oracle on S, and
+    outside S every copy holds the committed context."""
+    import oracle
+    _, g, inside = _subspace(oracle)
+    gi = g.astype(np.int64)
+    theta = visit["theta"]
+    context = oracle.bf16_bits_array(theta)
+    assert np.array_equal(visit["w_two_pairs0"], visit["w_member0"])
+    assert np.array_equal(visit["w_two_pairs1"], visit["w_member1"])
+    nid, sign = oracle.member_table(N, 1)[:2]
+    for i in (2, 3):
+        seed, s = int(visit["seeds"][nid[i]]), float(sign[i]) * SIGMA
+        ref, _ = oracle.perturb_at(g, theta[gi], seed, s, oracle.BF16)
+        scale = np.maximum(np.abs(theta[gi]), np.abs(np.float32(SIGMA) * oracle.noise(seed, g)))
+        got = visit[f"w_two_pairs{i}"]
+        assert_bf16_close(got[gi], ref.astype(np.uint16), scale)
+        assert np.array_equal(got[~inside], context[~inside])
