@@ -44,6 +44,7 @@ import argparse
 import hashlib
 import json
 import os
+import re
 import statistics
 import subprocess
 import sys
@@ -64,13 +65,13 @@ FALLBACK_HBM_GBS = 6800.0
 # subspaces of 2^28 parameters, where the writes still in L2 when the kernel ends are about
 # 2% of its traffic.
 NCU_TRAFFIC = {
-    "perturb_two_pairs": {"kernel": "elem_tiles_kernel<perturb_two_pairs,bf16>", "source_sha": "6adf05ff51bf21e3",
+    "perturb_two_pairs": {"kernel": "elem_tiles_kernel<perturb_two_pairs,bf16>", "source_sha": "2d16bf01a43641d5",
                           "bytes_per_elem": 11.782, "capture": "profiles/perturb_two_pairs_4b_slice.md",
                           "case": "two 2^28-parameter subspaces (--case 4b-slice-big)"},
-    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "6adf05ff51bf21e3",
+    "perturb_pair": {"kernel": "elem_tiles_kernel<perturb_pair,bf16>", "source_sha": "2d16bf01a43641d5",
                      "bytes_per_elem": 7.827, "capture": "profiles/perturb_pair_4b_slice.md",
                      "case": "two 2^28-parameter subspaces (--case 4b-slice-big --weights dual)"},
-    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "6adf05ff51bf21e3",
+    "perturb": {"kernel": "elem_tiles_kernel<perturb,bf16>", "source_sha": "2d16bf01a43641d5",
                 "bytes_per_elem": 5.862, "capture": "profiles/perturb_4b_slice.md",
                 "case": "two 2^28-parameter subspaces (--case 4b-slice-big --weights single)"},
 }
@@ -160,11 +161,15 @@ def measured_peaks():
 
 
 def source_sha():
-    """Hash of the sources the tile kernels compile from."""
+    """Hash of the code the tile kernels compile from: comments and blank space are
+    dropped first, so an edit to a comment keeps a capture valid and any code change
+    drops it."""
     h = hashlib.sha256()
     for name in ("es_kernels.cu", "copes_device.cuh", "copes_internal.h", "es_common.cuh", "normal_coeffs.h"):
-        with open(os.path.join(ROOT, "paper_2608_02391_gb300", "csrc", name), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2608_02391_gb300", "csrc", name)) as fh:
+            text = re.sub(r"/\*.*?\*/", "", fh.read(), flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        h.update("\n".join(line.strip() for line in text.splitlines() if line.strip()).encode())
     return h.hexdigest()[:16]
 
 

@@ -325,10 +325,11 @@ __device__ __forceinline__ void elem_tile_ragged(const ElemArgs &a, uint64_t b, 
 // the pair perturb takes G = 4 groups per step together (one tail vote for the four) at 4
 // resident blocks per SM (64 registers a thread): 0.603 ms against 0.631 ms for G = 8 one
 // group at a time at 3 blocks.  The two-pairs perturb takes G = 1 group (2 Philox blocks
-// per step, packed steps) at 4 blocks per SM (64 registers, no spill): 1.07 ms per
-// 503M-element subspace; G = 2 took 1.078 ms with scalar steps and 1.090 ms packed (52
-// bytes a thread spilled).  The other ops take G = 8 groups one at a time at 3 blocks per
-// SM (85 registers), which the plain perturb runs faster (0.532 against 0.544 ms).
+// per step, packed steps) at 4 blocks per SM (56 registers, no spill): 1.054 ms per
+// 503M-element subspace, against 1.088 ms at 5 blocks and, in an earlier form, 1.1-2.3%
+// more for G = 2 (scalar steps, or packed with 52 bytes a thread spilled).  The other ops
+// take G = 8 groups one at a time at 3 blocks per SM (85 registers), which the plain
+// perturb runs faster (0.532 against 0.544 ms).
 template <int OP>
 constexpr int elem_blocks_per_sm() { return OP == kOpPerturbPair || OP == kOpPerturbTwoPairs ? 4 : 3; }
 template <int OP>
