@@ -31,7 +31,7 @@ def _free_port():
         return s.getsockname()[1]
 
 
-def _setup(dual=False):
+def _setup(copies=1):
     import torch
     sys.path.insert(0, ROOT)
     from paper_2608_02391_gb300 import copes, es
@@ -40,7 +40,7 @@ def _setup(dual=False):
     gen.manual_seed(0)
     master = torch.empty(N_PARAMS, device="cuda").normal_(0.0, 0.02, generator=gen)
     w = master.to(torch.bfloat16)
-    arena = copes.Arena(w, master, w2=w.clone() if dual else None)
+    arena = copes.Arena(w, master, *[w.clone() for _ in range(copies - 1)])
     c = torch.empty(N_PARAMS, device="cuda").normal_(0.0, 1.0, generator=gen)
     layout = copes.Layout([N_PARAMS])
     subs = es.build_subspaces(layout, "contiguous", K, tile_size=4096)
@@ -72,20 +72,21 @@ def _oracle_check(torch, copes, arena, sub, k, cfg, rewards, f_gpu, idx, theta):
     got = arena.master[it].cpu().numpy()
     assert_update_close(got, exact, scale)
     commit = oracle.bf16_bits_array(got)
-    for w in (arena.w, arena.w2):
-        if w is not None:
-            assert np.array_equal(w.view(torch.int16)[it].cpu().numpy().view(np.uint16), commit)
+    for w in arena.copies:
+        assert np.array_equal(w.view(torch.int16)[it].cpu().numpy().view(np.uint16), commit)
 
 
-def _worker(rank, world, port, out, dual):
+def _worker(rank, world, port, out, copies):
     import torch.distributed as dist
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
     # a bounded collective timeout: a rank that fails ends its peer's next all-gather
     dist.init_process_group("gloo", rank=rank, world_size=world, timeout=datetime.timedelta(seconds=120))
     try:
-        torch, copes, es, arena, c, subs, cfg = _setup(dual)
-        # dual: each rank evaluates its antithetic pairs on two working copies
-        partner = es.Partner.second_copy(arena) if dual else None
+        torch, copes, es, arena, c, subs, cfg = _setup(copies)
+        # each rank evaluates its antithetic pairs on two working copies, or two pairs at a
+        # time on four
+        partner = {1: None, 2: es.Partner.second_copy, 4: es.Partner.four_copies}[copies]
+        partner = partner(arena) if partner else None
 
         def evaluate(i):  # the reward of the live perturbation: a linear objective
             return float((c * arena.live.float()).sum().item())
@@ -101,8 +102,8 @@ def _worker(rank, world, port, out, dual):
                                     rewards_out=rewards)
             if rank == 0:
                 _oracle_check(torch, copes, arena, subs[k], k, cfg, rewards, f.cpu().numpy(), idx, theta)
-        if dual:  # both copies hold the new context
-            assert torch.equal(arena.w.view(torch.int16), arena.w2.view(torch.int16))
+        for w in arena.copies[1:]:  # every copy holds the new context
+            assert torch.equal(arena.w.view(torch.int16), w.view(torch.int16))
         copes.check()
         digest = _digest(torch, arena)
         ref = None
@@ -123,12 +124,12 @@ def _worker(rank, world, port, out, dual):
         dist.destroy_process_group()
 
 
-@pytest.mark.parametrize("dual", [False, True])
-def test_two_ranks_match_the_oracle_and_one_process(dual):
+@pytest.mark.parametrize("copies", [1, 2, 4])
+def test_two_ranks_match_the_oracle_and_one_process(copies):
     ctx = mp.get_context("spawn")
     out = ctx.Queue()
     port = _free_port()
-    procs = [ctx.Process(target=_worker, args=(r, 2, port, out, dual)) for r in range(2)]
+    procs = [ctx.Process(target=_worker, args=(r, 2, port, out, copies)) for r in range(2)]
     for p in procs:
         p.start()
     res = sorted((out.get(timeout=600) for _ in procs), key=lambda t: t[0])
