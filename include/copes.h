@@ -168,7 +168,8 @@ enum { COPES_COEF_PAPER = 0, COPES_COEF_OPENAI = 1 };
 
 /* -------------------------------------------------------------------- host utilities */
 
-/* Version string of the library (static storage). */
+/* Version string of the library (static storage).  0.2 added copes_params.w3 / w4 and
+ * copes_perturb_two_pairs: callers built against 0.1's copes_params must be rebuilt. */
 const char *copes_version(void);
 
 /* Copies the calling thread's last error message into buf (NUL-terminated, truncated to

@@ -289,7 +289,7 @@ void copes::set_last_error(const char *message) { g_message = message; }
 
 extern "C" {
 
-const char *copes_version(void) { return "copes-gb300 0.1 (sm_103a)"; }
+const char *copes_version(void) { return "copes-gb300 0.2 (sm_103a)"; }
 
 int copes_last_error(char *buf, size_t len) {
   if (buf && len) {
