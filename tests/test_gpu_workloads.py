@@ -195,6 +195,58 @@ def test_layer_block_workloads_sampled(copes, name, visits):
     copes.check()
 
 
+def test_4b_visits_on_four_working_copies_as_benched(copes):
+    """The bench's 4B configuration: tile tables of 16,384 elements, members written two
+    pairs at a time into four working copies (es.round_robin_visit with
+    Partner.four_copies), restore, shaping and the fused update + commit to every copy.
+    Every member's live weights, the update and the commit are checked against the oracle
+    on sampled indices of the first and last layer blocks; after each visit the four
+    copies are bit-identical."""
+    from paper_2608_02391_gb300 import es
+    w = wl.workload("4b")
+    arena1, layout = make_arena(copes, w)
+    arena = copes.Arena(arena1.w, arena1.master, *[arena1.w.clone() for _ in range(3)])
+    partner = es.Partner.four_copies(arena)
+    cfg = es.ESConfig(n_members=w.n_members, sigma=w.sigma, alpha=w.alpha, shaping=w.shaping)
+    nid, sign, P = copes.member_table(w.n_members, copes.ANTITHETIC)
+    rewards = wl.reward_stream(w, 8)
+    rng = np.random.default_rng(9)
+    for k in (0, w.K - 1):
+        sub = copes.subspace_build(layout, copes.PART_TENSOR_GROUPS, w.K, k, group_of=w.group_of,
+                                   tile_size=copes.DEFAULT_TILE)
+        sample = sample_from_ranges(tile_ranges(sub), 2048, rng)
+        idx_t = torch.from_numpy(sample).cuda()
+        theta = arena.master[idx_t].cpu().numpy()
+        g = sample.astype(np.uint64)
+        seeds = copes.member_seeds(cfg.base_seed, 0, k, P)
+        s_k64 = es.sigma_k(cfg, layout.d_pad, sub.numel)  # the visit's sigma_k (a double)
+        s_k = float(np.float32(s_k64))  # as the kernels receive it
+        live = {}
+
+        def evaluate(i):  # the live copy's bits at the sample, as a rollout would read them
+            live[i] = arena.live.view(torch.int16)[idx_t].cpu().numpy().view(np.uint16)
+
+        r_dev = torch.from_numpy(rewards[k]).cuda()
+        f = es.round_robin_visit(arena, sub, k, 0, cfg, layout.d_pad, r_dev, evaluate=evaluate, partner=partner)
+        copes.check()
+        assert sorted(live) == list(range(w.n_members))
+        for i in range(w.n_members):
+            seed, s = int(seeds[nid[i]]), float(sign[i]) * s_k
+            ref_bits, _ = oracle.perturb_at(g, theta, seed, s, oracle.BF16)
+            scale = np.maximum(np.abs(theta), np.abs(np.float32(s_k) * oracle.noise(seed, g)))
+            assert_bf16_close(live[i], ref_bits.astype(np.uint16), scale)
+        f_ref = oracle.shape_fitness(rewards[k], SHAPE[w.shaping])
+        assert_fitness_close(f.cpu().numpy(), f_ref)
+        coef = np.float32(copes.step_coef(cfg.alpha, w.n_members, s_k64, cfg.convention))
+        _, exact, scale = oracle.update_at(g, theta, seeds, oracle.noise_weights(nid, sign, f_ref, P), coef)
+        got = arena.master[idx_t].cpu().numpy()
+        assert_update_close(got, exact, scale)
+        commit = oracle.bf16_bits_array(got)
+        for c in arena.copies:
+            assert np.array_equal(bf16_bits_of(c, sample), commit)
+            assert torch.equal(c.view(torch.int16), arena.w.view(torch.int16))
+
+
 def test_8b_type_groups_sampled(copes):
     w = wl.workload("8b")
     arena, layout = make_arena(copes, w)
