@@ -195,15 +195,17 @@ def test_layer_block_workloads_sampled(copes, name, visits):
     copes.check()
 
 
-def test_4b_visits_on_four_working_copies_as_benched(copes):
-    """The bench's 4B configuration: tile tables of 16,384 elements, members written two
+@pytest.mark.parametrize("name", ["0.5b", "4b"])
+def test_visits_on_four_working_copies_as_benched(copes, name):
+    """The bench's configuration of the layer-block workloads: tile tables of 16,384
+    elements, members written two
     pairs at a time into four working copies (es.round_robin_visit with
     Partner.four_copies), restore, shaping and the fused update + commit to every copy.
     Every member's live weights, the update and the commit are checked against the oracle
     on sampled indices of the first and last layer blocks; after each visit the four
     copies are bit-identical."""
     from paper_2608_02391_gb300 import es
-    w = wl.workload("4b")
+    w = wl.workload(name)
     arena1, layout = make_arena(copes, w)
     arena = copes.Arena(arena1.w, arena1.master, *[arena1.w.clone() for _ in range(3)])
     partner = es.Partner.four_copies(arena)
