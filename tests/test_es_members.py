@@ -1,6 +1,6 @@
-"""Host logic of es.perturb_members: which members are perturbed by copes_perturb_pair,
-which are copied in from the partner buffer, and which take a plain copes_perturb (no GPU:
-the three calls are recorded, not run)."""
+"""Host logic of es.perturb_members: which members are perturbed by copes_perturb_two_pairs
+or copes_perturb_pair, which are copied in from the partner buffer, and which take a plain
+copes_perturb (no GPU: the calls are recorded, not run)."""
 import numpy as np
 import pytest
 
@@ -14,6 +14,8 @@ def calls(monkeypatch):
     monkeypatch.setattr(copes, "perturb_pair",
                         lambda a, s, seed, ss, buf, base: log.append(("pair", seed, ss, base)))
     monkeypatch.setattr(copes, "perturb_partner", lambda a, s, buf, base: log.append(("partner", base)))
+    monkeypatch.setattr(copes, "perturb_two_pairs",
+                        lambda a, s, sa, sb, ss: log.append(("two_pairs", sa, sb, ss)))
     return log
 
 
@@ -69,3 +71,40 @@ def test_in_place_partner_evaluates_the_second_member_on_w2(calls):
     assert seen == [(0, "w"), (1, "w2"), (2, "w"), (3, "w2"), (4, "w"), (5, "w2")]
     assert calls == [("pair", 100, 0.5, 0), ("pair", 101, 0.5, 0), ("pair", 102, 0.5, 0)]
     assert arena.live == "w"
+
+
+def four_copy_run(members, n_members, kind=copes.SUBSPACE_TILES):
+    from types import SimpleNamespace
+    arena = SimpleNamespace(w="w", w2="w2", w3="w3", w4="w4", live="w")
+    sub = SimpleNamespace(kind=kind)
+    nid, sign, P = copes.member_table(n_members, copes.ANTITHETIC)
+    seeds = np.arange(100, 100 + P, dtype=np.uint64)
+    seen = []
+    es.perturb_members(arena, sub, members, nid, sign, seeds, 0.5, lambda i: seen.append((i, arena.live)),
+                       es.Partner(arena.w2, 0, True, True))
+    assert arena.live == "w"
+    return seen
+
+
+def test_four_copies_take_two_pairs_per_pass(calls):
+    """Members 4m .. 4m+3 are written by one two-pairs pass and evaluated on w, w2, w3, w4;
+    a pair left over at the end goes to w and w2."""
+    seen = four_copy_run(range(10), 10)
+    assert seen == [(0, "w"), (1, "w2"), (2, "w3"), (3, "w4"), (4, "w"), (5, "w2"), (6, "w3"), (7, "w4"),
+                    (8, "w"), (9, "w2")]
+    assert calls == [("two_pairs", 100, 101, 0.5), ("two_pairs", 102, 103, 0.5), ("pair", 104, 0.5, 0)]
+
+
+def test_four_copies_on_other_subspace_kinds_take_pairs(calls):
+    """The two-pairs kernel takes tile subspaces only: index-list and replay subspaces run
+    their pairs one at a time on w and w2."""
+    seen = four_copy_run(range(4), 4, kind=copes.SUBSPACE_INDICES)
+    assert seen == [(0, "w"), (1, "w2"), (2, "w"), (3, "w2")]
+    assert calls == [("pair", 100, 0.5, 0), ("pair", 101, 0.5, 0)]
+
+
+def test_four_copies_on_a_slice_that_splits_the_groups(calls):
+    """Members 3 .. 9 of 12: member 3 alone, then 4 .. 7 in one pass, then the pair 8, 9."""
+    seen = four_copy_run(range(3, 10), 12)
+    assert [i for i, _ in seen] == list(range(3, 10))
+    assert calls == [("perturb", 101, -0.5), ("two_pairs", 102, 103, 0.5), ("pair", 104, 0.5, 0)]
