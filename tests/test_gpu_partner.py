@@ -407,3 +407,22 @@ def test_visit_on_four_working_copies_is_bit_identical(copes, kind, n_members):
     assert t0 == t1 and len(t0) == 3 * n_members
     assert all(np.array_equal(bits(c), bits(a0.w)) for c in a1.copies)
     assert np.array_equal(a1.master.cpu().numpy().view(np.uint32), a0.master.cpu().numpy().view(np.uint32))
+
+
+def test_two_pairs_range_check_reports_without_faulting(copes):
+    """A tile past the arena's end: the two-pairs kernel skips it whole, writes no copy
+    there, and copes_check reports the device check; the valid tile is written."""
+    theta = theta_np(1000)
+    arena = quad_arena(copes, theta, torch.bfloat16)
+    before = [bits(c).copy() for c in arena.copies]
+    bad = copes.SubspaceHandle(copes.SUBSPACE_TILES,
+                               torch.tensor([[0, 100], [900, 5000]], dtype=torch.int64, device="cuda"), 0)
+    copes.perturb_two_pairs(arena, bad, 1, 2, 1e-3)
+    with pytest.raises(copes.CopesError) as e:
+        copes.check()
+    assert e.value.code == copes.ERR_DEVICE_CHECK
+    for c, b in zip(arena.copies, before):
+        got = bits(c)
+        assert np.array_equal(got[100:], b[100:])  # the bad tile was skipped whole
+        assert not np.array_equal(got[:100], b[:100])
+    copes.check()  # cleared
